@@ -1,0 +1,183 @@
+/*
+ * videomla.h -- C ABI of libvideomla.so: the latent KV cache and the
+ * absorbed-form Multi-Head Latent Attention of VideoMLA (arXiv 2605.30351)
+ * on one GB300 (sm_103a).
+ *
+ * Conventions for every entry point
+ *  - All tensors are caller-owned device memory (for example torch tensors
+ *    passed by data_ptr()). The library allocates no device memory, keeps no
+ *    per-cache state of its own and never synchronises the stream.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
+ *    NULL is the legacy default stream).
+ *  - bf16 = IEEE bfloat16 stored as 2 bytes. All arrays are dense, row-major,
+ *    with the last dimension contiguous, and start on a 16-byte boundary.
+ *  - Return 0 (MLA_OK) or a negative MLA_ERR_* code. Host-side validation
+ *    runs before any launch, so an error return means nothing was enqueued.
+ *    Faults the host cannot see (a position outside the RoPE table, a device
+ *    wait that ran out) are recorded in a device status word that
+ *    mla_device_status() reads; the kernel skips the offending work instead
+ *    of trapping.
+ */
+#ifndef VIDEOMLA_H_
+#define VIDEOMLA_H_
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MLA_OK 0
+#define MLA_ERR_ARG (-1)         /* null pointer, misaligned pointer, bad shape */
+#define MLA_ERR_UNSUPPORTED (-2) /* no kernel instance for this shape */
+#define MLA_ERR_RANGE (-3)       /* frame count or position outside the window/table */
+#define MLA_ERR_CUDA (-4)        /* launch or runtime error (see mla_last_cuda_error) */
+#define MLA_ERR_TIMEOUT (-5)     /* a bounded device-side wait ran out */
+
+/* cfg.flags */
+#define MLA_FLAG_NO_RMSNORM 1u   /* store c^KV = W_dkv x without RMSNorm (App. D.2 off) */
+#define MLA_FLAG_SIMT 2u         /* use the plain SIMT debug kernels (no tensor cores) */
+
+/*
+ * Shape of one VideoMLA attention layer (Sec. 3; App. D.2-D.4).
+ *  hidden          d, the model width (1536 for Wan2.1-1.3B)
+ *  heads           n_h (12)
+ *  head_dim        d_h = d_nope + d_rope (128); the score is divided by
+ *                  sqrt(head_dim) (Eq. score)
+ *  d_c             width of the shared KV latent c^KV (192)   (Eq. ckv)
+ *  d_r             width of the shared positional key k^R (32) (Eq. krope)
+ *  d_q             width of the query latent (768); informational here
+ *  rope_pairs_*    complex pairs per axis; 2*(t+h+w) must equal d_r (App. D.3)
+ *  rope_dim_*      band width D_a of each axis: pair i of axis a rotates with
+ *                  theta^(-2i/D_a), i.e. the highest-frequency bands of the
+ *                  backbone's per-axis split (44/42/42 for a 128-wide head);
+ *                  0 means D_a = 2 * rope_pairs_a
+ *  rope_theta      RoPE base (10000)
+ *  rope_table_len  positions per axis the table covers (1024, App. C.1)
+ *  tokens_per_frame T, tokens of one latent frame (30*52 = 1560, App. D.1)
+ *  window_frames   W, latent frames the ring holds (21, Sec. 1 / App. D.4)
+ *  batch           B, independent sequences, each with its own ring
+ *  rms_eps         RMSNorm epsilon (1e-6)
+ *  flags           MLA_FLAG_*
+ */
+typedef struct mla_config {
+  int hidden;
+  int heads;
+  int head_dim;
+  int d_c;
+  int d_r;
+  int d_q;
+  int rope_pairs_t, rope_pairs_h, rope_pairs_w;
+  int rope_dim_t, rope_dim_h, rope_dim_w;
+  double rope_theta;
+  int rope_table_len;
+  int tokens_per_frame;
+  int window_frames;
+  int batch;
+  float rms_eps;
+  unsigned flags;
+} mla_config;
+
+/*
+ * The sliding-window latent cache (App. D.4). Caller-owned device buffers:
+ *  c          bf16 [batch][window_frames*tokens_per_frame][d_c]   latent c^KV
+ *  kr         bf16 [batch][window_frames*tokens_per_frame][d_r]   rotated k^R
+ *  rope_table fp32 [rope_table_len][d_r/2][2] = (cos, sin) of position p
+ *             times the pair's frequency; fill it with mla_rope_table_fill()
+ *             and copy it to the device.
+ *  frames_written  number of latent frames appended so far (advanced by
+ *             mla_cache_append on the host; reset by mla_cache_reset).
+ * Token k of latent frame f lives in slot (f mod window_frames)*T + k
+ * (FIFO eviction, App. D.4). Slots of frames that were never written are
+ * not read.
+ */
+typedef struct mla_cache {
+  void* c;
+  void* kr;
+  const void* rope_table;
+  long long frames_written;
+  mla_config cfg;
+} mla_cache;
+
+/* Bytes of the host buffer mla_rope_table_fill writes (0 on a bad config). */
+unsigned long long mla_rope_table_bytes(const mla_config* cfg);
+
+/*
+ * Fill host_table (fp32 [rope_table_len][d_r/2][2]) with cos/sin of
+ * p * theta^(-2i/D_a) for every position p and pair (axis a, band i),
+ * computed in double and rounded once (Sec. 3.2, App. D.3).
+ * Returns MLA_ERR_ARG on a null pointer or an inconsistent config.
+ */
+int mla_rope_table_fill(const mla_config* cfg, float* host_table);
+
+/* Check a configuration without launching anything. */
+int mla_config_check(const mla_config* cfg);
+
+/*
+ * Zero both cache buffers and set frames_written = 0 (asynchronous memset
+ * on `stream`).
+ */
+int mla_cache_reset(mla_cache* cache, void* stream);
+
+/*
+ * Append n_frames latent frames (first_frame .. first_frame+n_frames-1) of
+ * token activations to the cache (Eqs. ckv and krope; App. D.2, D.4):
+ *     c = RMSNorm_gamma(W_dkv x)        -> cache.c  at the frame's slots
+ *     k = RoPE3D(W_kr x, pos)           -> cache.kr at the frame's slots
+ *  x        bf16 [batch][n_frames*T][hidden]
+ *  w_dkv    bf16 [d_c][hidden]        joint KV down-projection
+ *  gamma_kv bf16 [d_c] RMSNorm weight, or NULL for ones
+ *  w_kr     bf16 [d_r][hidden]        decoupled RoPE key projection
+ *  pos      int32 [batch][n_frames*T][3]  (t, h, w) of every token; each
+ *           coordinate must lie in [0, rope_table_len) (device-checked)
+ * The positional key is rotated here with the absolute positions given;
+ * the scores only depend on position differences, so this matches
+ * rotating at use with window-relative coordinates (Sec. 3.2, App. D.5).
+ * Rules: 1 <= n_frames <= window_frames (else MLA_ERR_RANGE);
+ * 0 <= first_frame <= frames_written <= first_frame + n_frames (no gap, and
+ * the range reaches the newest frame: extend the window or rewrite the
+ * current chunk, as each denoising step does). Afterwards
+ * frames_written = first_frame + n_frames.
+ */
+int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv,
+                     const void* gamma_kv, const void* w_kr, const int* pos,
+                     long long first_frame, int n_frames, void* stream);
+
+/*
+ * Absorbed-form attention of a query chunk against every valid slot of the
+ * window (Eq. score; App. E, Eqs. absorb-q and absorb-v):
+ *     s_hj  = (q_c,h . c_j + RoPE3D(q_r,h, q_pos) . k_j) / sqrt(head_dim)
+ *     o_h   = sum_j softmax_j(s_hj) c_j            (latent output, d_c wide)
+ *  q_c   bf16 [batch][Nq][heads][d_c]  absorbed content queries A_h^T c^Q
+ *  q_r   bf16 [batch][Nq][heads][d_r]  unrotated positional queries
+ *  q_pos int32 [batch][Nq][3]          query positions (device-checked)
+ *  o_lat bf16 [batch][Nq][heads][d_c]  output; the caller applies
+ *        B_h = W_O,h W_up,h^V to mix heads (Eq. absorb-v)
+ * Valid slots: the first min(frames_written, W)*T slots before the ring
+ * first wraps, all slots after. The query chunk is taken to be the newest
+ * chunk, so the chunk-causal mask (App. D.4) keeps every valid slot.
+ * MLA_ERR_ARG if no slot is valid or Nq < 1.
+ */
+int mla_attention_forward(const mla_cache* cache, const void* q_c,
+                          const void* q_r, const int* q_pos, int Nq,
+                          void* o_lat, void* stream);
+
+/* Human-readable name of a status code. */
+const char* mla_status_string(int status);
+
+/* The cudaError_t of the last MLA_ERR_CUDA return (0 if none). */
+int mla_last_cuda_error(void);
+
+/*
+ * Read (and, if clear != 0, reset) the device status word that kernels set
+ * when they skip work: MLA_OK, MLA_ERR_RANGE or MLA_ERR_TIMEOUT. The first
+ * error recorded wins. Synchronises the device.
+ */
+int mla_device_status(int* status, int clear);
+
+/* Library version, e.g. 100 for 0.1.0. */
+int mla_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VIDEOMLA_H_ */

@@ -1,0 +1,290 @@
+// C ABI of libvideomla.so: argument checks, the RoPE table, tensor-map
+// encoding and dispatch to the kernels. See include/videomla.h.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include <cudaTypedefs.h>
+
+#include "internal.h"
+#include "ptx_sm103.cuh"
+
+namespace vmla {
+namespace {
+
+__device__ int g_device_status = MLA_OK;
+
+thread_local int t_last_cuda_error = 0;
+
+constexpr int kMaxDevices = 64;
+int* g_status_ptr[kMaxDevices] = {nullptr};
+std::mutex g_mu;
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int* device_status_ptr() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+    g_status_ptr[dev] = static_cast<int*>(p);
+  }
+  return g_status_ptr[dev];
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  return g_encode;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int pairs_total(const mla_config& c) { return c.rope_pairs_t + c.rope_pairs_h + c.rope_pairs_w; }
+
+int axis_dim(const mla_config& c, int a) {
+  const int d = a == 0 ? c.rope_dim_t : (a == 1 ? c.rope_dim_h : c.rope_dim_w);
+  const int n = a == 0 ? c.rope_pairs_t : (a == 1 ? c.rope_pairs_h : c.rope_pairs_w);
+  return d > 0 ? d : 2 * n;
+}
+
+int check_config(const mla_config* c) {
+  if (!c) return MLA_ERR_ARG;
+  if (c->hidden <= 0 || c->heads <= 0 || c->head_dim <= 0 || c->d_c <= 0 || c->d_r < 0 ||
+      c->tokens_per_frame <= 0 || c->window_frames <= 0 || c->batch <= 0 ||
+      c->rope_table_len <= 0 || !(c->rope_theta > 0.0) || !(c->rms_eps >= 0.f))
+    return MLA_ERR_ARG;
+  if (c->rope_pairs_t < 0 || c->rope_pairs_h < 0 || c->rope_pairs_w < 0) return MLA_ERR_ARG;
+  if (2 * pairs_total(*c) != c->d_r) return MLA_ERR_ARG;
+  for (int a = 0; a < 3; ++a) {
+    const int n = a == 0 ? c->rope_pairs_t : (a == 1 ? c->rope_pairs_h : c->rope_pairs_w);
+    if (n > 0 && axis_dim(*c, a) < 2 * n) return MLA_ERR_ARG;
+  }
+  // every row must be a whole number of 16-byte chunks (vector stores, TMA strides)
+  if (c->d_c % 8 != 0 || c->d_r % 8 != 0 || c->hidden % 8 != 0) return MLA_ERR_ARG;
+  const long long slots = static_cast<long long>(c->tokens_per_frame) * c->window_frames;
+  if (slots > (1ll << 30)) return MLA_ERR_ARG;
+  return MLA_OK;
+}
+
+int fail_cuda(cudaError_t e) {
+  t_last_cuda_error = static_cast<int>(e);
+  return MLA_ERR_CUDA;
+}
+
+}  // namespace
+
+void set_last_cuda_error(cudaError_t e) { t_last_cuda_error = static_cast<int>(e); }
+
+bool encode_map_3d_bf16(CUtensorMap* map, const void* base, unsigned long long d0,
+                        unsigned long long d1, unsigned long long d2,
+                        unsigned long long stride1_bytes, unsigned long long stride2_bytes,
+                        unsigned b0, unsigned b1, CUtensorMapSwizzle swizzle) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {stride1_bytes, stride2_bytes};
+  const cuuint32_t box[3] = {b0, b1, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_map_2d_bf16(CUtensorMap* map, const void* base, unsigned long long d0,
+                        unsigned long long d1, unsigned long long stride1_bytes, unsigned b0,
+                        unsigned b1, CUtensorMapSwizzle swizzle) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {d0, d1};
+  const cuuint64_t strides[1] = {stride1_bytes};
+  const cuuint32_t box[2] = {b0, b1};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace vmla
+
+using namespace vmla;
+
+extern "C" {
+
+int mla_version(void) { return 100; }
+
+int mla_config_check(const mla_config* cfg) { return check_config(cfg); }
+
+unsigned long long mla_rope_table_bytes(const mla_config* cfg) {
+  if (check_config(cfg) != MLA_OK) return 0;
+  return static_cast<unsigned long long>(cfg->rope_table_len) * (cfg->d_r / 2) * 2 *
+         sizeof(float);
+}
+
+int mla_rope_table_fill(const mla_config* cfg, float* host_table) {
+  if (check_config(cfg) != MLA_OK || !host_table) return MLA_ERR_ARG;
+  const int np = cfg->d_r / 2;
+  // frequency of each pair: axis blocks t, h, w; band i of axis a -> theta^(-2i/D_a)
+  double freq[1024];
+  if (np > 1024) return MLA_ERR_ARG;
+  int k = 0;
+  for (int a = 0; a < 3; ++a) {
+    const int n = a == 0 ? cfg->rope_pairs_t : (a == 1 ? cfg->rope_pairs_h : cfg->rope_pairs_w);
+    const double D = static_cast<double>(axis_dim(*cfg, a));
+    for (int i = 0; i < n; ++i) freq[k++] = std::pow(cfg->rope_theta, -2.0 * i / D);
+  }
+  for (int pos = 0; pos < cfg->rope_table_len; ++pos)
+    for (int i = 0; i < np; ++i) {
+      const double ang = static_cast<double>(pos) * freq[i];
+      host_table[(static_cast<size_t>(pos) * np + i) * 2 + 0] = static_cast<float>(std::cos(ang));
+      host_table[(static_cast<size_t>(pos) * np + i) * 2 + 1] = static_cast<float>(std::sin(ang));
+    }
+  return MLA_OK;
+}
+
+int mla_cache_reset(mla_cache* cache, void* stream) {
+  if (!cache) return MLA_ERR_ARG;
+  const int rc = check_config(&cache->cfg);
+  if (rc != MLA_OK) return rc;
+  if (!cache->c || (!cache->kr && cache->cfg.d_r > 0)) return MLA_ERR_ARG;
+  const mla_config& c = cache->cfg;
+  const size_t slots = static_cast<size_t>(c.tokens_per_frame) * c.window_frames;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemsetAsync(cache->c, 0, slots * c.batch * c.d_c * 2, s);
+  if (e == cudaSuccess && c.d_r > 0) e = cudaMemsetAsync(cache->kr, 0, slots * c.batch * c.d_r * 2, s);
+  if (e != cudaSuccess) return fail_cuda(e);
+  cache->frames_written = 0;
+  return MLA_OK;
+}
+
+int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv, const void* gamma_kv,
+                     const void* w_kr, const int* pos, long long first_frame, int n_frames,
+                     void* stream) {
+  if (!cache) return MLA_ERR_ARG;
+  int rc = check_config(&cache->cfg);
+  if (rc != MLA_OK) return rc;
+  const mla_config& c = cache->cfg;
+  if (!cache->c || !cache->kr || !cache->rope_table || !x || !w_dkv || !w_kr || !pos)
+    return MLA_ERR_ARG;
+  if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(x) || !aligned16(w_dkv) ||
+      !aligned16(w_kr) || !aligned16(cache->rope_table) || (gamma_kv && !aligned16(gamma_kv)) ||
+      (reinterpret_cast<uintptr_t>(pos) & 3u))
+    return MLA_ERR_ARG;
+  if (n_frames < 1 || n_frames > c.window_frames) return MLA_ERR_RANGE;
+  if (first_frame < 0 || first_frame > cache->frames_written ||
+      first_frame + n_frames < cache->frames_written)
+    return MLA_ERR_ARG;
+  AppendArgs a;
+  a.x = x;
+  a.w_dkv = w_dkv;
+  a.gamma = gamma_kv;
+  a.w_kr = w_kr;
+  a.pos = pos;
+  a.rope = static_cast<const float*>(cache->rope_table);
+  a.c = cache->c;
+  a.kr = cache->kr;
+  a.batch = c.batch;
+  a.n_tok = n_frames * c.tokens_per_frame;
+  a.hidden = c.hidden;
+  a.d_c = c.d_c;
+  a.d_r = c.d_r;
+  a.slots = c.tokens_per_frame * c.window_frames;
+  a.tokens_per_frame = c.tokens_per_frame;
+  a.window_frames = c.window_frames;
+  a.first_frame = first_frame;
+  a.rope_len = c.rope_table_len;
+  a.pairs_t = c.rope_pairs_t;
+  a.pairs_h = c.rope_pairs_h;
+  a.use_rmsnorm = (c.flags & MLA_FLAG_NO_RMSNORM) ? 0 : 1;
+  a.eps = c.rms_eps;
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  rc = (c.flags & MLA_FLAG_SIMT) ? launch_append_simt(a) : launch_append_tc(a);
+  if (rc != MLA_OK) return rc;
+  cache->frames_written = first_frame + n_frames;
+  return MLA_OK;
+}
+
+int mla_attention_forward(const mla_cache* cache, const void* q_c, const void* q_r,
+                          const int* q_pos, int Nq, void* o_lat, void* stream) {
+  if (!cache) return MLA_ERR_ARG;
+  int rc = check_config(&cache->cfg);
+  if (rc != MLA_OK) return rc;
+  const mla_config& c = cache->cfg;
+  if (!cache->c || !cache->kr || !cache->rope_table || !q_c || !q_r || !q_pos || !o_lat)
+    return MLA_ERR_ARG;
+  if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(q_c) || !aligned16(q_r) ||
+      !aligned16(o_lat) || !aligned16(cache->rope_table) ||
+      (reinterpret_cast<uintptr_t>(q_pos) & 3u))
+    return MLA_ERR_ARG;
+  if (Nq < 1) return MLA_ERR_ARG;
+  const long long held = cache->frames_written < c.window_frames ? cache->frames_written
+                                                                  : c.window_frames;
+  const long long n_valid = held * c.tokens_per_frame;
+  if (n_valid < 1) return MLA_ERR_ARG;
+  const long long rows = static_cast<long long>(Nq) * c.heads;
+  if (rows > (1ll << 30)) return MLA_ERR_ARG;
+  AttnArgs a;
+  a.q_c = q_c;
+  a.q_r = q_r;
+  a.q_pos = q_pos;
+  a.rope = static_cast<const float*>(cache->rope_table);
+  a.c = cache->c;
+  a.kr = cache->kr;
+  a.o = o_lat;
+  a.batch = c.batch;
+  a.rows = static_cast<int>(rows);
+  a.heads = c.heads;
+  a.slots = c.tokens_per_frame * c.window_frames;
+  a.n_valid = static_cast<int>(n_valid);
+  a.d_c = c.d_c;
+  a.d_r = c.d_r;
+  a.rope_len = c.rope_table_len;
+  a.pairs_t = c.rope_pairs_t;
+  a.pairs_h = c.rope_pairs_h;
+  a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c.head_dim)));
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return (c.flags & MLA_FLAG_SIMT) ? launch_attention_simt(a) : launch_attention_tc(a);
+}
+
+const char* mla_status_string(int status) {
+  switch (status) {
+    case MLA_OK: return "ok";
+    case MLA_ERR_ARG: return "invalid argument";
+    case MLA_ERR_UNSUPPORTED: return "shape not supported by this kernel";
+    case MLA_ERR_RANGE: return "frame count or position out of range";
+    case MLA_ERR_CUDA: return "CUDA error";
+    case MLA_ERR_TIMEOUT: return "device wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int mla_last_cuda_error(void) { return t_last_cuda_error; }
+
+int mla_device_status(int* status, int clear) {
+  if (!status) return MLA_ERR_ARG;
+  int* p = device_status_ptr();
+  if (!p) return fail_cuda(cudaGetLastError());
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(status, p, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && clear) {
+    const int zero = MLA_OK;
+    e = cudaMemcpy(p, &zero, sizeof(int), cudaMemcpyHostToDevice);
+  }
+  return e == cudaSuccess ? MLA_OK : fail_cuda(e);
+}
+
+}  // extern "C"

@@ -1,0 +1,312 @@
+// Fused cache append on the sm_103a tensor cores.
+//
+// Paper: Eq. (ckv) c = W_dn^KV x, RMSNorm on c (App. D.2), Eq. (krope)
+// k = RoPE3D(W_R^K x), FIFO ring write (App. D.4). One CTA takes 128 tokens:
+//   warp 0     TMA producer: x tile [128 x 64] and the matching 64 columns of
+//              [W_dkv ; W_kr] ([d_c + d_r] x 64) per stage, SW128.
+//   warp 1     allocates TMEM; one lane issues tcgen05.mma into one
+//              [128 x (d_c + d_r)] fp32 accumulator (a single N = 224 MMA per
+//              K step at the paper's shape).
+//   warps 2-5  epilogue, thread i = token i: RMSNorm over the d_c columns in
+//              fp32, gamma, RoPE3D on the d_r columns, bf16, 16-byte stores
+//              into the token's ring slot (f mod W) * T + k.
+#include <cmath>
+
+#include "internal.h"
+#include "ptx_sm103.cuh"
+
+namespace vmla {
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+
+template <int DC, int DR>
+struct AppendShape {
+  static constexpr int N = DC + DR;
+  static constexpr bool kSplitN = N > 256;  // then two MMAs: c part and k part
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = N * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kFit = (232448 - 1024 - kBarBytes) / kStageBytes;
+  static constexpr int kStages = kFit > 6 ? 6 : kFit;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
+  static constexpr uint32_t kTmemCols = N <= 256 ? 256 : 512;
+  static_assert(DC % 32 == 0 && DR % 32 == 0 && DC <= 256 && DR <= 64, "shape");
+  static_assert(N <= 512, "accumulator must fit in TMEM");
+  static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
+  static_assert(kStages >= 2, "smem");
+};
+
+struct AppendKParams {
+  const __nv_bfloat16* gamma;
+  const int* pos;
+  const float2* rope;
+  __nv_bfloat16* c;
+  __nv_bfloat16* kr;
+  int n_tok, k_blocks, slots, T, W;
+  long long first_frame;
+  int rope_len, pairs_t, pairs_h, use_rmsnorm;
+  float eps;
+  int* status;
+};
+
+template <int DC, int DR>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_append_tc_kernel(const __grid_constant__ CUtensorMap tm_x,
+                         const __grid_constant__ CUtensorMap tm_wc,
+                         const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
+  using S = AppendShape<DC, DR>;
+  constexpr int NST = S::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align_smem_1024(smem_raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NST * S::kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + NST;
+  uint64_t* acc_full = bars + 2 * NST;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.y;
+  const int row0 = blockIdx.x * kBM;
+  const WaitCtx wc{abort_flag, p.status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(acc_full, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, S::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_x);
+      tma_prefetch_desc(&tm_wc);
+      tma_prefetch_desc(&tm_wk);
+      int issued = 0;
+      for (int kb = 0; kb < p.k_blocks; ++kb) {
+        const int st = kb % NST;
+        if (kb >= NST && !mbar_wait(&empty[st], ((kb / NST) - 1) & 1, wc)) break;
+        uint8_t* a = smem + st * S::kStageBytes;
+        uint8_t* bm = a + S::kABytes;
+        mbar_arrive_expect_tx(&full[st], S::kStageBytes);
+        tma_load_3d(a, &tm_x, &full[st], kb * kBK, row0, b);
+        tma_load_2d(bm, &tm_wc, &full[st], kb * kBK, 0);
+        tma_load_2d(bm + DC * 128, &tm_wk, &full[st], kb * kBK, 0);
+        issued = kb + 1;
+      }
+      if (*abort_flag)
+        for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
+          mbar_wait_drain(&full[u % NST], (u / NST) & 1, p.status);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = true;
+      for (int kb = 0; kb < p.k_blocks; ++kb) {
+        const int st = kb % NST;
+        if (!mbar_wait(&full[st], (kb / NST) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t aa = smem_u32(smem + st * S::kStageBytes);
+        const uint32_t ba = aa + S::kABytes;
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k) {
+          const uint32_t acc = (kb | k) != 0 ? 1u : 0u;
+          const uint64_t ad = sdesc(aa + k * 32, 16, 1024, kSw128);
+          if constexpr (!S::kSplitN) {
+            constexpr uint32_t idesc = idesc_bf16_f32(kBM, S::N, false, false);
+            umma_ss(tmem, ad, sdesc(ba + k * 32, 16, 1024, kSw128), idesc, acc);
+          } else {
+            constexpr uint32_t idesc_c = idesc_bf16_f32(kBM, DC, false, false);
+            constexpr uint32_t idesc_k = idesc_bf16_f32(kBM, DR, false, false);
+            umma_ss(tmem, ad, sdesc(ba + k * 32, 16, 1024, kSw128), idesc_c, acc);
+            umma_ss(tmem + DC, ad, sdesc(ba + DC * 128 + k * 32, 16, 1024, kSw128), idesc_k, acc);
+          }
+        }
+        umma_commit(&empty[st]);
+      }
+      umma_commit(acc_full);
+      if (!ok) mbar_wait_drain(acc_full, 0, p.status);
+    }
+    __syncwarp();
+  } else {
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t t_row = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    const int n = row0 + r;
+    const bool row_ok = n < p.n_tok;
+    if (mbar_wait(acc_full, 0, wc) && !*abort_flag) {
+      tc_fence_after();
+      // pass 1: mean square of c over d_c (fp32)
+      float ss = 0.f;
+#pragma unroll 1
+      for (int cb = 0; cb < DC / 32; ++cb) {
+        uint32_t v[32];
+        tmem_ld32(t_row + cb * 32, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float f = __uint_as_float(v[i]);
+          ss = fmaf(f, f, ss);
+        }
+      }
+      const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
+      const long long f = p.first_frame + n / p.T;
+      const long long slot = (f % p.W) * p.T + n % p.T;
+      uint4* cdst = reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC);
+      // pass 2: gamma * c / rms -> bf16 -> ring slot
+#pragma unroll 1
+      for (int cb = 0; cb < DC / 32; ++cb) {
+        uint32_t v[32];
+        tmem_ld32(t_row + cb * 32, v);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float g0 = 1.f, g1 = 1.f;
+          if (p.gamma) {
+            g0 = __bfloat162float(p.gamma[cb * 32 + 2 * i]);
+            g1 = __bfloat162float(p.gamma[cb * 32 + 2 * i + 1]);
+          }
+          pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]) * inv * g0,
+                              __uint_as_float(v[2 * i + 1]) * inv * g1);
+        }
+        if (row_ok) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            cdst[cb * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        }
+      }
+      // positional key: RoPE3D at the token's (t, h, w)
+      int pa[3] = {0, 0, 0};
+      if (row_ok) {
+        const int* pp = p.pos + (static_cast<size_t>(b) * p.n_tok + n) * 3;
+        pa[0] = __ldg(pp);
+        pa[1] = __ldg(pp + 1);
+        pa[2] = __ldg(pp + 2);
+#pragma unroll
+        for (int a = 0; a < 3; ++a)
+          if (pa[a] < 0 || pa[a] >= p.rope_len) {
+            record_status(p.status, MLA_ERR_RANGE);
+            pa[a] = 0;
+          }
+      }
+      uint4* kdst = reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR);
+#pragma unroll 1
+      for (int cb = 0; cb < DR / 32; ++cb) {
+        uint32_t v[32];
+        tmem_ld32(t_row + DC + cb * 32, v);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int pr = cb * 16 + i;
+          const int ps = pr < p.pairs_t ? pa[0] : (pr < p.pairs_t + p.pairs_h ? pa[1] : pa[2]);
+          const float2 cs = __ldg(p.rope + static_cast<size_t>(ps) * (DR / 2) + pr);
+          const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
+          pk[i] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
+        }
+        if (row_ok) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            kdst[cb * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, S::kTmemCols);
+  }
+}
+
+template <int DC, int DR>
+int launch_tc(const AppendArgs& a) {
+  using S = AppendShape<DC, DR>;
+  CUtensorMap tm_x, tm_wc, tm_wk;
+  const unsigned long long H = a.hidden, n_tok = a.n_tok;
+  if (!encode_map_3d_bf16(&tm_x, a.x, H, n_tok, a.batch, H * 2, n_tok * H * 2, kBK, kBM,
+                          CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_2d_bf16(&tm_wc, a.w_dkv, H, DC, H * 2, kBK, DC, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_2d_bf16(&tm_wk, a.w_kr, H, DR, H * 2, kBK, DR, CU_TENSOR_MAP_SWIZZLE_128B))
+    return MLA_ERR_CUDA;
+  auto kern = mla_append_tc_kernel<DC, DR>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  AppendKParams kp;
+  kp.gamma = static_cast<const __nv_bfloat16*>(a.gamma);
+  kp.pos = a.pos;
+  kp.rope = reinterpret_cast<const float2*>(a.rope);
+  kp.c = static_cast<__nv_bfloat16*>(a.c);
+  kp.kr = static_cast<__nv_bfloat16*>(a.kr);
+  kp.n_tok = a.n_tok;
+  kp.k_blocks = a.hidden / kBK;
+  kp.slots = a.slots;
+  kp.T = a.tokens_per_frame;
+  kp.W = a.window_frames;
+  kp.first_frame = a.first_frame;
+  kp.rope_len = a.rope_len;
+  kp.pairs_t = a.pairs_t;
+  kp.pairs_h = a.pairs_h;
+  kp.use_rmsnorm = a.use_rmsnorm;
+  kp.eps = a.eps;
+  kp.status = a.status;
+  const dim3 grid((a.n_tok + kBM - 1) / kBM, a.batch);
+  kern<<<grid, kThreads, S::kSmemBytes, a.stream>>>(tm_x, tm_wc, tm_wk, kp);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  return MLA_OK;
+}
+
+}  // namespace
+
+int launch_append_tc(const AppendArgs& a) {
+  if (a.hidden % kBK != 0) return MLA_ERR_UNSUPPORTED;
+  if (a.d_r == 32) {
+    switch (a.d_c) {
+      case 64: return launch_tc<64, 32>(a);
+      case 128: return launch_tc<128, 32>(a);
+      case 192: return launch_tc<192, 32>(a);
+      case 256: return launch_tc<256, 32>(a);
+      default: break;
+    }
+  } else if (a.d_r == 64) {
+    switch (a.d_c) {
+      case 64: return launch_tc<64, 64>(a);
+      case 128: return launch_tc<128, 64>(a);
+      case 192: return launch_tc<192, 64>(a);
+      case 256: return launch_tc<256, 64>(a);
+      default: break;
+    }
+  }
+  return MLA_ERR_UNSUPPORTED;
+}
+
+}  // namespace vmla

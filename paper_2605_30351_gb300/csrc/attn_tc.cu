@@ -1,0 +1,428 @@
+// Absorbed-form MLA attention on the sm_103a tensor cores (tcgen05 + TMEM + TMA).
+//
+// Paper: Eq. (score) and App. E (Eqs. absorb-q, absorb-v). Every query row is
+// one (token, head) pair; all rows of a batch element score the SAME cached
+// latents, so the n_h heads simply stack along M and each KV tile is loaded
+// once per 128 rows:
+//     S   = [q_c | RoPE(q_r)] . [c | k]^T          K = d_c + d_r (224)
+//     P   = exp2(S * log2(e)/sqrt(d_h) - m)        online, fp32
+//     O  += P . c                                  N = d_c (192), latent output
+// One CTA owns 128 rows (one TMEM lane each) and walks the window in blocks
+// of 128 keys:
+//   warp 0     TMA producer: q_c tile once, then [c | k] tiles into a ring of
+//              shared-memory stages (no multicast).
+//   warp 1     allocates TMEM; one lane issues every tcgen05.mma:
+//              S_j = Q K_j^T into TMEM buffer j%2 (SS form), then
+//              O += P_{j-1} V_{j-1} with P read from TMEM (TS form).
+//   warps 2-5  rotate q_r into the Q tile, then the online softmax: thread i
+//              owns row i, reads S_j from TMEM, writes P_j (bf16) over S_j's
+//              first half, rescales O in TMEM only when its running max grows
+//              by more than 2^8, and finally writes O / l as bf16.
+// The V operand is the first d_c columns of the same K tile read MN-major,
+// so the cache is never expanded into per-head keys or values.
+#include <cmath>
+
+#include "internal.h"
+#include "ptx_sm103.cuh"
+
+namespace vmla {
+namespace {
+
+constexpr int kBM = 128;       // rows per CTA = TMEM lanes
+constexpr int kBN = 128;       // keys per block
+constexpr int kThreads = 192;  // 6 warps
+constexpr float kRescaleLog2 = 8.0f;
+
+template <int DC, int DR>
+struct AttnShape {
+  static constexpr int DK = DC + DR;
+  static constexpr int kTileBytes = kBM * DK * 2;  // the Q tile and one KV stage (kBM == kBN)
+  static constexpr int kKrOff = DC * kBM * 2;      // byte offset of the d_r columns in a tile
+  static constexpr int kBarBytes = 256;
+  static constexpr int kSmemCap = 232448;
+  static constexpr int kFit = (kSmemCap - 1024 - kBarBytes - kTileBytes) / kTileBytes;
+  static constexpr int kStages = kFit > 4 ? 4 : kFit;
+  static constexpr int kSmemBytes = 1024 + kTileBytes * (1 + kStages) + kBarBytes;
+  static constexpr int kTmemO = 2 * kBN;
+  static constexpr uint32_t kTmemCols = 512;
+  static constexpr uint32_t kKrSw = DR == 32 ? kSw64 : kSw128;
+  static constexpr uint32_t kKrRow = DR * 2;     // bytes per row of the d_r block
+  static constexpr uint32_t kKrSbo = 8 * kKrRow;  // one 8-row swizzle atom
+  static constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
+  static constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, DC, false, true);
+  static_assert(kBM == kBN, "the Q tile and a KV stage share one size");
+  static_assert(DC % 64 == 0 && DC >= 64 && DC <= 256, "d_c: multiple of 64 up to 256");
+  static_assert(DR == 32 || DR == 64, "d_r: 32 or 64");
+  static_assert(kTmemO + DC <= 512, "two S buffers plus O must fit in 512 TMEM columns");
+  static_assert(kStages >= 2, "at least two KV stages must fit in shared memory");
+  static_assert(kTileBytes % 1024 == 0 && kKrOff % 1024 == 0, "swizzle-atom alignment");
+};
+
+struct AttnKParams {
+  const __nv_bfloat16* q_r;
+  const int* q_pos;
+  const float2* rope;
+  __nv_bfloat16* o;
+  int rows, heads, n_valid, rope_len, pairs_t, pairs_h;
+  float scale_log2;
+  int* status;
+};
+
+template <int DC, int DR>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_qc,
+                       const __grid_constant__ CUtensorMap tm_c,
+                       const __grid_constant__ CUtensorMap tm_kr, const AttnKParams p) {
+  using S = AttnShape<DC, DR>;
+  constexpr int NST = S::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align_smem_1024(smem_raw);
+  uint8_t* sQ = smem;
+  uint8_t* sKV = smem + S::kTileBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + NST * S::kTileBytes);
+  uint64_t* q_tma_full = bars + 0;
+  uint64_t* q_rot_ready = bars + 1;
+  uint64_t* kv_full = bars + 2;
+  uint64_t* kv_empty = kv_full + NST;
+  uint64_t* s_full = kv_empty + NST;
+  uint64_t* p_full = s_full + 2;
+  uint64_t* pv_done = p_full + 2;
+  uint64_t* mma_drain = pv_done + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.y;
+  const int row0 = blockIdx.x * kBM;
+  const int nblk = (p.n_valid + kBN - 1) / kBN;
+  const WaitCtx wc{abort_flag, p.status};
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_tma_full, 1);
+    mbar_init(q_rot_ready, kBM);
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], kBM);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_init(mma_drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, S::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_qc);
+      tma_prefetch_desc(&tm_c);
+      tma_prefetch_desc(&tm_kr);
+      mbar_arrive_expect_tx(q_tma_full, DC * kBM * 2);
+      for (int cb = 0; cb < DC / 64; ++cb)
+        tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, cb * 64, row0, b);
+      int issued = 0;
+      for (int j = 0; j < nblk; ++j) {
+        const int st = j % NST;
+        if (j >= NST && !mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, wc)) break;
+        uint8_t* kv = sKV + st * S::kTileBytes;
+        mbar_arrive_expect_tx(&kv_full[st], S::kTileBytes);
+        for (int cb = 0; cb < DC / 64; ++cb)
+          tma_load_3d(kv + cb * 16384, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
+        tma_load_3d(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b);
+        issued = j + 1;
+      }
+      if (*abort_flag) {  // let every copy this CTA started land before exit
+        mbar_wait_drain(q_tma_full, 0, p.status);
+        for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
+          mbar_wait_drain(&kv_full[u % NST], (u / NST) & 1, p.status);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(q_tma_full, 0, wc) && mbar_wait(q_rot_ready, 0, wc);
+      tc_fence_after();
+      const uint32_t qa = smem_u32(sQ);
+      auto issue_pv = [&](int i) -> bool {
+        if (!mbar_wait(&p_full[i & 1], (i >> 1) & 1, wc)) return false;
+        tc_fence_after();
+        const int st = i % NST;
+        const uint32_t va = smem_u32(sKV) + st * S::kTileBytes;
+        const uint32_t a_p = tmem + (i & 1) * kBN;  // bf16 P over S_i's first 64 columns
+#pragma unroll
+        for (int s = 0; s < kBN / 16; ++s)
+          umma_ts(tmem + S::kTmemO, a_p + s * 8, sdesc(va + s * 2048, 16384, 1024, kSw128),
+                  S::kIdescPV, (i > 0 || s > 0) ? 1u : 0u);
+        umma_commit(&kv_empty[st]);
+        umma_commit(&pv_done[i & 1]);
+        return true;
+      };
+      for (int j = 0; ok && j < nblk; ++j) {
+        const int st = j % NST;
+        if (!mbar_wait(&kv_full[st], (j / NST) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t ka = smem_u32(sKV) + st * S::kTileBytes;
+        const uint32_t d_s = tmem + (j & 1) * kBN;
+#pragma unroll
+        for (int cb = 0; cb < DC / 64; ++cb)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_ss(d_s, sdesc(qa + cb * 16384 + k * 32, 16, 1024, kSw128),
+                    sdesc(ka + cb * 16384 + k * 32, 16, 1024, kSw128), S::kIdescQK,
+                    (cb | k) != 0 ? 1u : 0u);
+#pragma unroll
+        for (int k = 0; k < DR / 16; ++k)
+          umma_ss(d_s, sdesc(qa + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw),
+                  sdesc(ka + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw), S::kIdescQK, 1u);
+        umma_commit(&s_full[j & 1]);
+        if (j > 0 && !issue_pv(j - 1)) ok = false;
+      }
+      if (ok) ok = issue_pv(nblk - 1);
+      if (!ok) {  // wait for every MMA already issued before TMEM is freed
+        umma_commit(mma_drain);
+        mbar_wait_drain(mma_drain, 0, p.status);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------ softmax (warps 2..5)
+    const int quarter = warp & 3;  // TMEM lane quarter this warp may access
+    const int r = quarter * 32 + lane;
+    const uint32_t t_lane = static_cast<uint32_t>(quarter * 32) << 16;
+    const int grow = row0 + r;
+    const bool row_ok = grow < p.rows;
+
+    // q_r -> RoPE3D(q_r) in bf16, written into the Q tile's d_r block using
+    // the same 16-byte-chunk swizzle the TMA would apply.
+    {
+      uint32_t w[DR / 2];
+#pragma unroll
+      for (int i = 0; i < DR / 2; ++i) w[i] = 0u;
+      if (row_ok) {
+        const uint4* src = reinterpret_cast<const uint4*>(
+            p.q_r + (static_cast<size_t>(b) * p.rows + grow) * DR);
+#pragma unroll
+        for (int i = 0; i < DR / 8; ++i) {
+          const uint4 v = __ldg(src + i);
+          w[4 * i + 0] = v.x;
+          w[4 * i + 1] = v.y;
+          w[4 * i + 2] = v.z;
+          w[4 * i + 3] = v.w;
+        }
+        const int nq = p.rows / p.heads;
+        const int* pp = p.q_pos + (static_cast<size_t>(b) * nq + grow / p.heads) * 3;
+        int pa[3] = {__ldg(pp), __ldg(pp + 1), __ldg(pp + 2)};
+#pragma unroll
+        for (int a = 0; a < 3; ++a)
+          if (pa[a] < 0 || pa[a] >= p.rope_len) {
+            record_status(p.status, MLA_ERR_RANGE);
+            pa[a] = 0;
+          }
+#pragma unroll
+        for (int i = 0; i < DR / 2; ++i) {
+          const int pos = i < p.pairs_t ? pa[0] : (i < p.pairs_t + p.pairs_h ? pa[1] : pa[2]);
+          const float2 cs = __ldg(p.rope + static_cast<size_t>(pos) * (DR / 2) + i);
+          const float x0 = bf16_lo(w[i]), x1 = bf16_hi(w[i]);
+          w[i] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
+        }
+      }
+      uint8_t* krow = sQ + S::kKrOff + r * S::kKrRow;
+#pragma unroll
+      for (int c = 0; c < DR / 8; ++c) {
+        const int phys = DR == 32 ? (c ^ ((r >> 1) & 3)) : (c ^ (r & 7));
+        *reinterpret_cast<uint4*>(krow + phys * 16) =
+            make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(q_rot_ready);
+    }
+
+    float m_run = -INFINITY;
+    float l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nblk; ++j) {
+      if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, wc)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t t_s = tmem + t_lane + (j & 1) * kBN;
+      uint32_t sr[kBN];
+#pragma unroll
+      for (int c = 0; c < kBN / 32; ++c)
+        tmem_ld32(t_s + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
+      tmem_wait_ld();
+      float sv[kBN];
+#pragma unroll
+      for (int c = 0; c < kBN; ++c) sv[c] = __uint_as_float(sr[c]);
+      const int valid = p.n_valid - j * kBN;
+      if (valid < kBN) {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c)
+          if (c >= valid) sv[c] = -INFINITY;
+      }
+      float mx = sv[0];
+#pragma unroll
+      for (int c = 1; c < kBN; ++c) mx = fmaxf(mx, sv[c]);
+      const float m_blk = mx * p.scale_log2;
+      if (j == 0) {
+        m_run = m_blk;
+      } else {
+        const bool need = m_blk > m_run + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          // O is only touched once PV_{j-1} has landed.
+          if (!mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, wc)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          float alpha = 1.f;
+          if (need) {
+            alpha = ex2_approx(m_run - m_blk);
+            m_run = m_blk;
+          }
+          l_run *= alpha;
+#pragma unroll 1
+          for (int c = 0; c < DC / 32; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * alpha);
+            tmem_st32(tmem + t_lane + S::kTmemO + c * 32, ov);
+          }
+          tmem_wait_st();
+        }
+      }
+      const float neg_m = -m_run;
+      float l0 = 0.f, l1 = 0.f;
+      uint32_t pk[kBN / 2];
+#pragma unroll
+      for (int i = 0; i < kBN / 2; ++i) {
+        const float p0 = ex2_approx(fmaf(sv[2 * i], p.scale_log2, neg_m));
+        const float p1 = ex2_approx(fmaf(sv[2 * i + 1], p.scale_log2, neg_m));
+        l0 += p0;
+        l1 += p1;
+        pk[i] = pack_bf16x2(p0, p1);
+      }
+      l_run += l0 + l1;
+#pragma unroll
+      for (int c = 0; c < kBN / 64; ++c)
+        tmem_st32(t_s + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[c * 32]));
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&p_full[j & 1]);
+    }
+
+    if (ok && mbar_wait(&pv_done[(nblk - 1) & 1], ((nblk - 1) >> 1) & 1, wc)) {
+      tc_fence_after();
+      const float inv_l = 1.f / l_run;
+      uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC);
+#pragma unroll 1
+      for (int c = 0; c < DC / 32; ++c) {
+        uint32_t ov[32];
+        tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          pk[i] = pack_bf16x2(__uint_as_float(ov[2 * i]) * inv_l,
+                              __uint_as_float(ov[2 * i + 1]) * inv_l);
+        if (row_ok) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            dst[c * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, S::kTmemCols);
+  }
+}
+
+template <int DC, int DR>
+int launch_tc(const AttnArgs& a) {
+  using S = AttnShape<DC, DR>;
+  CUtensorMap tm_qc, tm_c, tm_kr;
+  const unsigned long long rows = a.rows, slots = a.slots;
+  if (!encode_map_3d_bf16(&tm_qc, a.q_c, DC, rows, a.batch, DC * 2ull, rows * DC * 2ull, 64,
+                          kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_3d_bf16(&tm_c, a.c, DC, a.n_valid, a.batch, DC * 2ull, slots * DC * 2ull, 64,
+                          kBN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_3d_bf16(&tm_kr, a.kr, DR, a.n_valid, a.batch, DR * 2ull, slots * DR * 2ull, DR,
+                          kBN,
+                          DR == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
+    return MLA_ERR_CUDA;
+  auto kern = mla_attn_tc_kernel<DC, DR>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  AttnKParams kp;
+  kp.q_r = static_cast<const __nv_bfloat16*>(a.q_r);
+  kp.q_pos = a.q_pos;
+  kp.rope = reinterpret_cast<const float2*>(a.rope);
+  kp.o = static_cast<__nv_bfloat16*>(a.o);
+  kp.rows = a.rows;
+  kp.heads = a.heads;
+  kp.n_valid = a.n_valid;
+  kp.rope_len = a.rope_len;
+  kp.pairs_t = a.pairs_t;
+  kp.pairs_h = a.pairs_h;
+  kp.scale_log2 = a.scale_log2;
+  kp.status = a.status;
+  const dim3 grid((a.rows + kBM - 1) / kBM, a.batch);
+  kern<<<grid, kThreads, S::kSmemBytes, a.stream>>>(tm_qc, tm_c, tm_kr, kp);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  return MLA_OK;
+}
+
+}  // namespace
+
+int launch_attention_tc(const AttnArgs& a) {
+  if (a.d_r == 32) {
+    switch (a.d_c) {
+      case 64: return launch_tc<64, 32>(a);
+      case 128: return launch_tc<128, 32>(a);
+      case 192: return launch_tc<192, 32>(a);
+      case 256: return launch_tc<256, 32>(a);
+      default: break;
+    }
+  } else if (a.d_r == 64) {
+    switch (a.d_c) {
+      case 64: return launch_tc<64, 64>(a);
+      case 128: return launch_tc<128, 64>(a);
+      case 192: return launch_tc<192, 64>(a);
+      default: break;
+    }
+  }
+  return MLA_ERR_UNSUPPORTED;
+}
+
+}  // namespace vmla

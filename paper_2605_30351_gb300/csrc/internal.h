@@ -1,0 +1,67 @@
+// Host-side interface between the C ABI (api.cu) and the kernel files.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "videomla.h"
+
+namespace vmla {
+
+// One attention launch: every (token, head) row of the chunk against the
+// valid slots of its batch element's window.
+struct AttnArgs {
+  const void* q_c;      // bf16 [B][rows][d_c]   rows = Nq * heads
+  const void* q_r;      // bf16 [B][rows][d_r]
+  const int* q_pos;     // int32 [B][Nq][3]
+  const float* rope;    // fp32 [L][d_r/2][2]
+  const void* c;        // bf16 [B][slots][d_c]
+  const void* kr;       // bf16 [B][slots][d_r]
+  void* o;              // bf16 [B][rows][d_c]
+  int batch, rows, heads, slots, n_valid;
+  int d_c, d_r, rope_len, pairs_t, pairs_h;
+  float scale_log2;     // log2(e) / sqrt(head_dim)
+  int* status;          // device status word
+  cudaStream_t stream;
+};
+
+// One append launch: n_tok tokens per batch element into their ring slots.
+struct AppendArgs {
+  const void* x;        // bf16 [B][n_tok][hidden]
+  const void* w_dkv;    // bf16 [d_c][hidden]
+  const void* gamma;    // bf16 [d_c] or nullptr
+  const void* w_kr;     // bf16 [d_r][hidden]
+  const int* pos;       // int32 [B][n_tok][3]
+  const float* rope;    // fp32 [L][d_r/2][2]
+  void* c;              // bf16 [B][slots][d_c]
+  void* kr;             // bf16 [B][slots][d_r]
+  int batch, n_tok, hidden, d_c, d_r, slots;
+  int tokens_per_frame, window_frames;
+  long long first_frame;
+  int rope_len, pairs_t, pairs_h;
+  int use_rmsnorm;
+  float eps;
+  int* status;
+  cudaStream_t stream;
+};
+
+// Each launcher returns MLA_OK, MLA_ERR_UNSUPPORTED or MLA_ERR_CUDA.
+int launch_attention_tc(const AttnArgs& a);
+int launch_attention_simt(const AttnArgs& a);
+int launch_append_tc(const AppendArgs& a);
+int launch_append_simt(const AppendArgs& a);
+
+// Shared by the launchers: cuTensorMapEncodeTiled fetched from the driver.
+// Encodes a rank-3 bf16 tiled map over [d2][d1][d0] (d0 contiguous) with
+// strides in bytes for dims 1 and 2 and a box of (b0, b1, 1).
+bool encode_map_3d_bf16(CUtensorMap* map, const void* base, unsigned long long d0,
+                        unsigned long long d1, unsigned long long d2,
+                        unsigned long long stride1_bytes, unsigned long long stride2_bytes,
+                        unsigned b0, unsigned b1, CUtensorMapSwizzle swizzle);
+bool encode_map_2d_bf16(CUtensorMap* map, const void* base, unsigned long long d0,
+                        unsigned long long d1, unsigned long long stride1_bytes, unsigned b0,
+                        unsigned b1, CUtensorMapSwizzle swizzle);
+
+void set_last_cuda_error(cudaError_t e);
+
+}  // namespace vmla

@@ -1,0 +1,217 @@
+"""ctypes binding of libvideomla.so (include/videomla.h), same names as the C ABI.
+
+Argument marshalling only: every step of the cache append and of the
+attention runs in the library's CUDA kernels. PyTorch supplies device memory
+and streams. There is no fallback: if the library is missing or a call
+fails, these functions raise.
+"""
+
+import ctypes
+import os
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libvideomla.so")
+
+MLA_OK = 0
+MLA_ERR_ARG = -1
+MLA_ERR_UNSUPPORTED = -2
+MLA_ERR_RANGE = -3
+MLA_ERR_CUDA = -4
+MLA_ERR_TIMEOUT = -5
+
+MLA_FLAG_NO_RMSNORM = 1
+MLA_FLAG_SIMT = 2
+
+# Every symbol include/videomla.h declares.
+EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
+           "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
+           "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
+
+
+class mla_config(ctypes.Structure):
+    _fields_ = [
+        ("hidden", ctypes.c_int), ("heads", ctypes.c_int), ("head_dim", ctypes.c_int),
+        ("d_c", ctypes.c_int), ("d_r", ctypes.c_int), ("d_q", ctypes.c_int),
+        ("rope_pairs_t", ctypes.c_int), ("rope_pairs_h", ctypes.c_int),
+        ("rope_pairs_w", ctypes.c_int),
+        ("rope_dim_t", ctypes.c_int), ("rope_dim_h", ctypes.c_int), ("rope_dim_w", ctypes.c_int),
+        ("rope_theta", ctypes.c_double), ("rope_table_len", ctypes.c_int),
+        ("tokens_per_frame", ctypes.c_int), ("window_frames", ctypes.c_int),
+        ("batch", ctypes.c_int), ("rms_eps", ctypes.c_float), ("flags", ctypes.c_uint),
+    ]
+
+
+class mla_cache(ctypes.Structure):
+    _fields_ = [
+        ("c", ctypes.c_void_p), ("kr", ctypes.c_void_p), ("rope_table", ctypes.c_void_p),
+        ("frames_written", ctypes.c_longlong), ("cfg", mla_config),
+    ]
+
+
+class MlaError(RuntimeError):
+    def __init__(self, fn, code, lib):
+        self.code = code
+        msg = lib.mla_status_string(code).decode()
+        if code == MLA_ERR_CUDA:
+            msg += f" (cudaError {lib.mla_last_cuda_error()})"
+        super().__init__(f"{fn} failed: {msg} [{code}]")
+
+
+_lib = None
+
+
+def load():
+    """Load the in-tree library once; raise if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, VP, I, LL = ctypes.POINTER, ctypes.c_void_p, ctypes.c_int, ctypes.c_longlong
+    lib.mla_rope_table_bytes.argtypes = [P(mla_config)]
+    lib.mla_rope_table_bytes.restype = ctypes.c_ulonglong
+    lib.mla_rope_table_fill.argtypes = [P(mla_config), P(ctypes.c_float)]
+    lib.mla_config_check.argtypes = [P(mla_config)]
+    lib.mla_cache_reset.argtypes = [P(mla_cache), VP]
+    lib.mla_cache_append.argtypes = [P(mla_cache), VP, VP, VP, VP, VP, LL, I, VP]
+    lib.mla_attention_forward.argtypes = [P(mla_cache), VP, VP, VP, I, VP, VP]
+    lib.mla_status_string.argtypes = [I]
+    lib.mla_status_string.restype = ctypes.c_char_p
+    lib.mla_last_cuda_error.argtypes = []
+    lib.mla_device_status.argtypes = [P(I), I]
+    lib.mla_version.argtypes = []
+    for name in ("mla_rope_table_fill", "mla_config_check", "mla_cache_reset", "mla_cache_append",
+                 "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
+                 "mla_version"):
+        getattr(lib, name).restype = I
+    _lib = lib
+    return lib
+
+
+def _check(fn, code):
+    if code != MLA_OK:
+        raise MlaError(fn, code, load())
+
+
+def make_config(w, flags=0):
+    """mla_config from a synth.Workload-like object."""
+    return mla_config(
+        hidden=w.hidden, heads=w.heads, head_dim=w.head_dim, d_c=w.d_c, d_r=w.d_r, d_q=w.d_q,
+        rope_pairs_t=w.rope_pairs[0], rope_pairs_h=w.rope_pairs[1], rope_pairs_w=w.rope_pairs[2],
+        rope_dim_t=w.rope_axis_dims[0], rope_dim_h=w.rope_axis_dims[1],
+        rope_dim_w=w.rope_axis_dims[2], rope_theta=w.rope_theta,
+        rope_table_len=w.rope_table_len, tokens_per_frame=w.tokens_per_frame,
+        window_frames=w.window_frames, batch=w.batch, rms_eps=w.rms_eps, flags=flags)
+
+
+def mla_config_check(cfg):
+    return load().mla_config_check(ctypes.byref(cfg))
+
+
+def mla_rope_table_fill(cfg):
+    """The RoPE cos/sin table as a float32 NumPy array [L, d_r/2, 2]."""
+    lib = load()
+    nbytes = lib.mla_rope_table_bytes(ctypes.byref(cfg))
+    if nbytes == 0:
+        raise MlaError("mla_rope_table_bytes", MLA_ERR_ARG, lib)
+    out = np.empty((cfg.rope_table_len, cfg.d_r // 2, 2), dtype=np.float32)
+    _check("mla_rope_table_fill",
+           lib.mla_rope_table_fill(ctypes.byref(cfg),
+                                   out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))))
+    return out
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t, dtype, shape, name):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class LatentCache:
+    """Device buffers of one layer's sliding-window latent cache + the C struct.
+
+    c  bf16 [B, W*T, d_c]; kr bf16 [B, W*T, d_r]; rope fp32 [L, d_r/2, 2].
+    """
+
+    def __init__(self, cfg, device="cuda"):
+        self.cfg = cfg
+        slots = cfg.tokens_per_frame * cfg.window_frames
+        self.c = torch.zeros(cfg.batch, slots, cfg.d_c, dtype=torch.bfloat16, device=device)
+        self.kr = torch.zeros(cfg.batch, slots, cfg.d_r, dtype=torch.bfloat16, device=device)
+        self.rope = torch.from_numpy(mla_rope_table_fill(cfg)).to(device)
+        self.struct = mla_cache(c=self.c.data_ptr(), kr=self.kr.data_ptr(),
+                                rope_table=self.rope.data_ptr(), frames_written=0, cfg=cfg)
+
+    @property
+    def frames_written(self):
+        return self.struct.frames_written
+
+    @frames_written.setter
+    def frames_written(self, v):
+        self.struct.frames_written = int(v)
+
+    @property
+    def slots(self):
+        return self.cfg.tokens_per_frame * self.cfg.window_frames
+
+    def n_valid(self):
+        held = min(self.frames_written, self.cfg.window_frames)
+        return held * self.cfg.tokens_per_frame
+
+
+def mla_cache_reset(cache, stream=None):
+    _check("mla_cache_reset",
+           load().mla_cache_reset(ctypes.byref(cache.struct), _stream_ptr(stream)))
+
+
+def mla_cache_append(cache, x, w_dkv, gamma_kv, w_kr, pos, first_frame, n_frames, stream=None):
+    cfg = cache.cfg
+    n_tok = n_frames * cfg.tokens_per_frame
+    bf = torch.bfloat16
+    args = (
+        _dev(x, bf, (cfg.batch, n_tok, cfg.hidden), "x"),
+        _dev(w_dkv, bf, (cfg.d_c, cfg.hidden), "w_dkv"),
+        None if gamma_kv is None else _dev(gamma_kv, bf, (cfg.d_c,), "gamma_kv"),
+        _dev(w_kr, bf, (cfg.d_r, cfg.hidden), "w_kr"),
+        _dev(pos, torch.int32, (cfg.batch, n_tok, 3), "pos"),
+    )
+    _check("mla_cache_append",
+           load().mla_cache_append(ctypes.byref(cache.struct), *args, int(first_frame),
+                                   int(n_frames), _stream_ptr(stream)))
+
+
+def mla_attention_forward(cache, q_c, q_r, q_pos, o_lat, stream=None):
+    cfg = cache.cfg
+    Nq = q_c.shape[1]
+    bf = torch.bfloat16
+    args = (
+        _dev(q_c, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "q_c"),
+        _dev(q_r, bf, (cfg.batch, Nq, cfg.heads, cfg.d_r), "q_r"),
+        _dev(q_pos, torch.int32, (cfg.batch, Nq, 3), "q_pos"),
+    )
+    out = _dev(o_lat, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "o_lat")
+    _check("mla_attention_forward",
+           load().mla_attention_forward(ctypes.byref(cache.struct), *args, int(Nq), out,
+                                        _stream_ptr(stream)))
+
+
+def mla_device_status(clear=True):
+    st = ctypes.c_int(0)
+    _check("mla_device_status", load().mla_device_status(ctypes.byref(st), int(bool(clear))))
+    return st.value

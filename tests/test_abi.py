@@ -1,0 +1,90 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every symbol the header declares, validates arguments before any launch, and
+its RoPE table matches the oracle's frequencies."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import mla_oracle as O
+from paper_2605_30351_gb300 import synth
+from paper_2605_30351_gb300 import videomla as V
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "videomla.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(mla_[a-z_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol():
+    lib = V.load()
+    names = declared_functions()
+    assert set(names) == set(V.EXPORTS), names
+    for n in names:
+        assert hasattr(lib, n), n
+    assert lib.mla_version() >= 100
+
+
+def test_struct_layout_matches_header():
+    # 12 ints, a double, 4 ints, a float, an unsigned (natural C alignment)
+    assert ctypes.sizeof(V.mla_config) == 80
+    assert V.mla_config.rope_theta.offset == 48
+    # three pointers, a long long, the config
+    assert ctypes.sizeof(V.mla_cache) == 112
+    assert V.mla_cache.cfg.offset == 32
+
+
+def test_config_validation():
+    w = synth.workload("wan")
+    cfg = V.make_config(w)
+    assert V.mla_config_check(cfg) == V.MLA_OK
+    bad = V.make_config(w)
+    bad.rope_pairs_t = 7                      # 2*(7+5+5) != 32
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    bad = V.make_config(w)
+    bad.d_c = 100                             # rows not 16-byte multiples
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    bad = V.make_config(w)
+    bad.rope_dim_h = 4                        # band width narrower than its pairs
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    bad = V.make_config(w)
+    bad.window_frames = 0
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+
+
+def test_null_arguments_rejected_before_launch():
+    lib = V.load()
+    w = synth.workload("tiny")
+    cache = V.mla_cache(cfg=V.make_config(w))
+    assert lib.mla_cache_append(ctypes.byref(cache), None, None, None, None, None, 0, 1,
+                                None) == V.MLA_ERR_ARG
+    assert lib.mla_attention_forward(ctypes.byref(cache), None, None, None, 1, None,
+                                     None) == V.MLA_ERR_ARG
+    assert lib.mla_cache_reset(None, None) == V.MLA_ERR_ARG
+    # n_frames beyond the window is a range error (checked before pointers are used)
+    fake = ctypes.c_void_p(1 << 20)
+    cache = V.mla_cache(c=fake, kr=fake, rope_table=fake, cfg=V.make_config(w))
+    assert lib.mla_cache_append(ctypes.byref(cache), fake, fake, None, fake, fake, 0,
+                                w.window_frames + 1, None) == V.MLA_ERR_RANGE
+    # misaligned pointer
+    odd = ctypes.c_void_p((1 << 20) + 2)
+    assert lib.mla_cache_append(ctypes.byref(cache), odd, fake, None, fake, fake, 0, 1,
+                                None) == V.MLA_ERR_ARG
+    assert lib.mla_status_string(V.MLA_ERR_RANGE).decode().startswith("frame count")
+
+
+@pytest.mark.parametrize("name", ["tiny", "wan"])
+def test_rope_table_matches_oracle_frequencies(name):
+    w = synth.workload(name)
+    tab = V.mla_rope_table_fill(V.make_config(w))
+    assert tab.shape == (w.rope_table_len, w.d_r // 2, 2)
+    inv, _axis = O.rope_inv_freq(O.RopeSpec(w.rope_pairs, w.rope_axis_dims, w.rope_theta))
+    pos = np.arange(w.rope_table_len)[:, None]
+    np.testing.assert_allclose(tab[..., 0], np.cos(pos * inv), rtol=0, atol=2e-7)
+    np.testing.assert_allclose(tab[..., 1], np.sin(pos * inv), rtol=0, atol=2e-7)

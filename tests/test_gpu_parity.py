@@ -1,0 +1,326 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 oracle on
+the same seeded inputs. Tolerance from the specification of this path:
+max-abs <= 2e-2 and relative L2 <= 1e-2 for floating point; ring-buffer
+indexing bit-exact."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import mla_oracle as O
+from paper_2605_30351_gb300 import synth
+from paper_2605_30351_gb300 import videomla as V
+
+pytestmark = pytest.mark.gpu
+
+MAX_ABS = 2e-2
+REL_L2 = 1e-2
+
+
+def assert_close(got, ref, max_abs=MAX_ABS, rel_l2=REL_L2, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite output"
+    d = got - ref
+    ma = float(np.max(np.abs(d))) if d.size else 0.0
+    rl = float(np.linalg.norm(d) / max(np.linalg.norm(ref), 1e-30))
+    assert ma <= max_abs and rl <= rel_l2, f"{what}: max_abs={ma:.3e} rel_l2={rl:.3e}"
+    return ma, rl
+
+
+def f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def spec_of(w):
+    return O.RopeSpec(w.rope_pairs, w.rope_axis_dims, w.rope_theta)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    V.load()
+    V.mla_device_status(clear=True)
+    yield
+    assert V.mla_device_status(clear=True) == V.MLA_OK
+
+
+def run_chunks(w, weights, chunks, flags=0, seed=100):
+    """Append `chunks` = [(first_frame, n_frames), ...] on the GPU and in the oracle."""
+    cfg = V.make_config(w, flags)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    oc = O.OracleCache(w.batch, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r)
+    dev = {k: v.cuda() for k, v in weights.items()}
+    for i, (first, n) in enumerate(chunks):
+        x = synth.draw_tokens(w, n * w.tokens_per_frame, seed + i)
+        pos = synth.grid_positions(w, first, n)
+        V.mla_cache_append(cache, x.cuda(), dev["w_dkv"], dev["gamma_kv"], dev["w_kr"],
+                           pos.cuda(), first, n)
+        O.cache_append(oc, f64(x), f64(weights["w_dkv"]), f64(weights["w_kr"]), pos.numpy(),
+                       first, n, gamma=f64(weights["gamma_kv"]), eps=w.rms_eps,
+                       use_rmsnorm=not (flags & V.MLA_FLAG_NO_RMSNORM), spec=spec_of(w))
+    torch.cuda.synchronize()
+    assert cache.frames_written == oc.frames_written
+    return cache, oc
+
+
+def small(name="tiny", **kw):
+    return synth.workload(name, **kw)
+
+
+# ------------------------------------------------------------------ append
+@pytest.mark.parametrize("flags", [0, V.MLA_FLAG_SIMT])
+def test_append_parity_tiny(flags):
+    w = small()
+    weights = synth.draw_layer_weights(w, seed=1)
+    cache, oc = run_chunks(w, weights, [(0, 1), (1, 1), (2, 1), (3, 1)], flags)
+    valid = oc.valid_slots()
+    assert_close(f64(cache.c)[:, valid], oc.c[:, valid], what="c")
+    assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what="k_rope")
+
+
+def test_append_parity_ragged_batch2_wrap():
+    # T = 100 tokens per frame (not a multiple of 128), batch 2, ring wraps
+    w = small(grid_h=10, grid_w=10, window_frames=5, batch=2, rope_pairs=(6, 5, 5))
+    weights = synth.draw_layer_weights(w, seed=2)
+    cache, oc = run_chunks(w, weights, [(0, 3), (3, 3), (3, 3), (6, 2)])
+    valid = oc.valid_slots()
+    assert len(valid) == 5 * 100
+    assert_close(f64(cache.c)[:, valid], oc.c[:, valid], what="c")
+    assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what="k_rope")
+
+
+def test_ring_bit_exact():
+    """One-hot projections, no RMSNorm, positions at zero: every appended
+    value is an input value, so slot contents must match bit for bit."""
+    w = small(grid_h=6, grid_w=7, window_frames=4, batch=2)
+    cfg = V.make_config(w, V.MLA_FLAG_NO_RMSNORM)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    d, dc, dr = w.hidden, w.d_c, w.d_r
+    w_dkv = torch.zeros(dc, d, dtype=torch.bfloat16)
+    w_dkv[torch.arange(dc), torch.arange(dc)] = 1
+    w_kr = torch.zeros(dr, d, dtype=torch.bfloat16)
+    w_kr[torch.arange(dr), dc + torch.arange(dr)] = 1
+    T = w.tokens_per_frame
+    frames = {}
+    schedule = [(0, 2), (2, 2), (4, 1), (5, 3), (8, 3), (8, 3), (11, 2)]
+    for i, (first, n) in enumerate(schedule):
+        x = synth.draw_tokens(w, n * T, 500 + i)
+        pos = torch.zeros(w.batch, n * T, 3, dtype=torch.int32)
+        V.mla_cache_append(cache, x.cuda(), w_dkv.cuda(), None, w_kr.cuda(), pos.cuda(), first, n)
+        for k in range(n):
+            frames[first + k] = x[:, k * T:(k + 1) * T]
+    torch.cuda.synchronize()
+    c_bits = cache.c.cpu().view(torch.int16)
+    k_bits = cache.kr.cpu().view(torch.int16)
+    for f in O.window_frames(cache.frames_written, w.window_frames):
+        s0 = O.ring_slot(f, 0, T, w.window_frames)
+        xb = frames[f].view(torch.int16)
+        assert torch.equal(c_bits[:, s0:s0 + T], xb[:, :, :dc]), f
+        assert torch.equal(k_bits[:, s0:s0 + T], xb[:, :, dc:dc + dr]), f
+
+
+# --------------------------------------------------------------- attention
+def upload_cache(w, seed, frames_written, flags=0):
+    """Fill a cache with seeded rows (not produced by the GPU) for attention tests."""
+    cfg = V.make_config(w, flags)
+    cache = V.LatentCache(cfg)
+    c, k = synth.draw_cache_rows(w, w.slots, seed)
+    cache.c.copy_(c)
+    cache.kr.copy_(k)
+    cache.frames_written = frames_written
+    return cache, f64(c), f64(k)
+
+
+def oracle_latent(w, q_c, q_r, q_pos, c, k, n_valid, rows=None):
+    out = []
+    for b in range(w.batch):
+        qc, qr, qp = f64(q_c[b]), f64(q_r[b]), q_pos[b].numpy()
+        if rows is not None:
+            tok = rows // w.heads
+            o = O.latent_attention(qc[tok], qr[tok], qp[tok], c[b, :n_valid], k[b, :n_valid],
+                                   w.head_dim, spec_of(w))
+            out.append(o[np.arange(len(rows)), rows % w.heads])
+        else:
+            out.append(O.latent_attention(qc, qr, qp, c[b, :n_valid], k[b, :n_valid],
+                                          w.head_dim, spec_of(w)))
+    return np.stack(out)
+
+
+@pytest.mark.parametrize("flags", [0, V.MLA_FLAG_SIMT])
+@pytest.mark.parametrize("case", [
+    dict(grid_h=8, grid_w=8, window_frames=4, fw=4, nq=64),     # tiny: 768 rows, 256 keys
+    dict(grid_h=10, grid_w=10, window_frames=5, fw=3, nq=50),   # ragged: 300 keys, 600 rows
+    dict(grid_h=9, grid_w=7, window_frames=3, fw=7, nq=63),     # wrapped ring, 189 keys
+])
+def test_attention_parity(case, flags):
+    case = dict(case)
+    fw, nq = case.pop("fw"), case.pop("nq")
+    w = small(batch=2, **case)
+    cache, c, k = upload_cache(w, 7, fw, flags)
+    q_c, q_r = synth.draw_queries(w, nq, 8)
+    q_pos = synth.grid_positions(w, max(fw - 1, 0), 1)[:, :nq].contiguous()
+    o = torch.empty(w.batch, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    ref = oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid())
+    assert_close(f64(o), ref, what="o_lat")
+
+
+@pytest.mark.parametrize("d_c,d_r,pairs", [
+    (64, 32, (4, 6, 6)), (128, 32, (6, 5, 5)), (256, 32, (6, 5, 5)),
+    (64, 64, (12, 10, 10)), (128, 64, (12, 10, 10)), (192, 64, (12, 10, 10)),
+])
+def test_attention_latent_sweep(d_c, d_r, pairs):
+    w = small(d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=(44, 42, 42) if d_r == 32
+              else (64, 64, 64), grid_h=10, grid_w=13, window_frames=3, batch=1)
+    cache, c, k = upload_cache(w, 11, 3)
+    q_c, q_r = synth.draw_queries(w, 40, 12)
+    q_pos = synth.grid_positions(w, 2, 1)[:, :40].contiguous()
+    o = torch.empty(1, 40, w.heads, d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    ref = oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid())
+    assert_close(f64(o), ref, what=f"o_lat d_c={d_c} d_r={d_r}")
+
+
+def test_attention_dc512_simt():
+    w = small(d_c=512, d_r=32, grid_h=6, grid_w=6, window_frames=3, batch=1)
+    cache, c, k = upload_cache(w, 13, 3, V.MLA_FLAG_SIMT)
+    q_c, q_r = synth.draw_queries(w, 20, 14)
+    q_pos = synth.grid_positions(w, 2, 1)[:, :20].contiguous()
+    o = torch.empty(1, 20, w.heads, 512, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    assert_close(f64(o), oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid()), what="d_c=512")
+
+
+def test_tc_matches_simt_wan_rows():
+    """Tensor-core and SIMT kernels agree at the full Wan-1.3B layer shape."""
+    w = synth.workload("wan")
+    cache, c, k = upload_cache(w, 21, w.window_frames)
+    q_c, q_r = synth.draw_queries(w, w.chunk_tokens, 22)
+    q_pos = synth.grid_positions(w, 18, 3)
+    args = (q_c.cuda(), q_r.cuda(), q_pos.cuda())
+    o_tc = torch.empty(1, w.chunk_tokens, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, *args, o_tc)
+    cache.struct.cfg.flags = V.MLA_FLAG_SIMT
+    o_simt = torch.empty_like(o_tc)
+    V.mla_attention_forward(cache, *args, o_simt)
+    torch.cuda.synchronize()
+    assert_close(f64(o_tc), f64(o_simt), what="tc vs simt")
+
+
+def test_attention_wan_sampled_rows():
+    """Full Wan-1.3B shape (4680 x 12 rows, 32760 keys), oracle on sampled rows."""
+    w = synth.workload("wan")
+    cache, c, k = upload_cache(w, 31, w.window_frames)
+    q_c, q_r = synth.draw_queries(w, w.chunk_tokens, 32)
+    q_pos = synth.grid_positions(w, 18, 3)
+    o = torch.empty(1, w.chunk_tokens, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(0)
+    rows = np.sort(rng.choice(w.chunk_tokens * w.heads, 96, replace=False))
+    rows = np.concatenate([rows, [0, w.chunk_tokens * w.heads - 1]])
+    ref = oracle_latent(w, q_c, q_r, q_pos, c, k, w.slots, rows=rows)
+    got = f64(o).reshape(1, -1, w.d_c)[:, rows]
+    assert_close(got, ref, what="wan sampled")
+
+
+def test_append_then_attention_chain():
+    """Each side runs its own append then attention: end-to-end latent output."""
+    w = small(grid_h=10, grid_w=12, window_frames=4, chunk_frames=2, batch=2)
+    weights = synth.draw_layer_weights(w, seed=41)
+    cache, oc = run_chunks(w, weights, [(0, 2), (2, 2), (4, 2)])
+    q_c, q_r = synth.draw_queries(w, 2 * w.tokens_per_frame, 42)
+    q_pos = synth.grid_positions(w, 4, 2)
+    o = torch.empty(w.batch, q_c.shape[1], w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    valid = oc.valid_slots()
+    ref = np.stack([O.latent_attention(f64(q_c[b]), f64(q_r[b]), q_pos[b].numpy(),
+                                       oc.c[b, valid], oc.kr[b, valid], w.head_dim, spec_of(w),
+                                       key_frames=oc.frame_of_slot[valid], query_last_frame=5)
+                    for b in range(w.batch)])
+    assert_close(f64(o), ref, what="chain")
+
+
+def test_rollout_positions_to_960():
+    """Batch 4, ring wrapped many times, temporal positions near 960."""
+    w = small(grid_h=12, grid_w=13, window_frames=21, chunk_frames=3, batch=4,
+              rope_pairs=(6, 5, 5))
+    weights = synth.draw_layer_weights(w, seed=51)
+    cfg = V.make_config(w)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    dev = {k: v.cuda() for k, v in weights.items()}
+    T = w.tokens_per_frame
+    # frames 0 .. 938 with cheap device-side activations (evicted before the check)
+    xz = torch.randn(w.batch, 3 * T, w.hidden, device="cuda").to(torch.bfloat16)
+    for first in range(0, 939, 3):
+        pos = synth.grid_positions(w, first, 3).cuda()
+        V.mla_cache_append(cache, xz, dev["w_dkv"], dev["gamma_kv"], dev["w_kr"], pos, first, 3)
+    oc = O.OracleCache(w.batch, T, w.window_frames, w.d_c, w.d_r)
+    oc.frames_written = 939
+    for i, first in enumerate(range(939, 960, 3)):     # the 7 chunks that stay in the window
+        x = synth.draw_tokens(w, 3 * T, 600 + i)
+        pos = synth.grid_positions(w, first, 3)
+        V.mla_cache_append(cache, x.cuda(), dev["w_dkv"], dev["gamma_kv"], dev["w_kr"],
+                           pos.cuda(), first, 3)
+        O.cache_append(oc, f64(x), f64(weights["w_dkv"]), f64(weights["w_kr"]), pos.numpy(),
+                       first, 3, gamma=f64(weights["gamma_kv"]), eps=w.rms_eps, spec=spec_of(w))
+    assert cache.frames_written == 960
+    valid = oc.valid_slots()
+    assert len(valid) == w.slots
+    assert_close(f64(cache.c)[:, valid], oc.c[:, valid], what="c at t~960")
+    assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what="k_rope at t~960")
+    q_c, q_r = synth.draw_queries(w, 3 * T, 61)
+    q_pos = synth.grid_positions(w, 957, 3)
+    o = torch.empty(w.batch, 3 * T, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    rows = np.arange(0, 3 * T * w.heads, 37)
+    ref = np.stack([O.latent_attention(f64(q_c[b]), f64(q_r[b]), q_pos[b].numpy(),
+                                       oc.c[b, valid], oc.kr[b, valid], w.head_dim,
+                                       spec_of(w)).reshape(-1, w.d_c)[rows]
+                    for b in range(w.batch)])
+    assert_close(f64(o).reshape(w.batch, -1, w.d_c)[:, rows], ref, what="rollout o_lat")
+
+
+# ------------------------------------------------------------ error paths
+def test_position_out_of_table_sets_device_status():
+    w = small()
+    cfg = V.make_config(w)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    weights = {k: v.cuda() for k, v in synth.draw_layer_weights(w, 3).items()}
+    x = synth.draw_tokens(w, w.tokens_per_frame, 4).cuda()
+    pos = synth.grid_positions(w, 0, 1).cuda()
+    pos[0, 5, 0] = w.rope_table_len          # one coordinate past the table
+    V.mla_cache_append(cache, x, weights["w_dkv"], weights["gamma_kv"], weights["w_kr"], pos, 0, 1)
+    assert V.mla_device_status(clear=True) == V.MLA_ERR_RANGE
+    assert V.mla_device_status(clear=True) == V.MLA_OK
+
+
+def test_host_argument_errors():
+    w = small()
+    cfg = V.make_config(w)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    q_c, q_r = synth.draw_queries(w, 8, 1)
+    q_pos = synth.grid_positions(w, 0, 1)[:, :8].contiguous()
+    o = torch.empty(1, 8, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(V.MlaError) as e:       # empty window
+        V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    assert e.value.code == V.MLA_ERR_ARG
+    weights = {k: v.cuda() for k, v in synth.draw_layer_weights(w, 3).items()}
+    x = synth.draw_tokens(w, w.tokens_per_frame, 4).cuda()
+    pos = synth.grid_positions(w, 2, 1).cuda()
+    with pytest.raises(V.MlaError) as e:       # a gap: frame 2 before frames 0, 1
+        V.mla_cache_append(cache, x, weights["w_dkv"], None, weights["w_kr"], pos, 2, 1)
+    assert e.value.code == V.MLA_ERR_ARG
