@@ -1,0 +1,424 @@
+"""Benchmark of one VideoMLA layer-chunk on GB300: cache append + absorbed MLA
+attention at the Wan2.1-1.3B shape (4680-query chunk, 32760-key window,
+12 heads, d_c = 192, d_r = 32, batch 1), through the C ABI.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One step = mla_cache_append of the current 3-frame chunk + mla_attention_forward
+of that chunk against the full 21-frame window (one layer, one denoising step).
+Prints one JSON line (rank 0). Multi-GPU runs are independent replicas
+(weak scaling): the path has no exchange step.
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2605_30351_gb300 import synth  # noqa: E402
+
+METRIC = "MLA attention TFLOP/s & % bf16 peak; ms per chunk per layer at Wan-1.3B shape"
+UNIT = "TFLOP/s"
+N_SETS = 4  # rotating input sets: 4 x 76 MB > 129 MB L2, so no set is L2-resident
+PROFILES = os.path.join(ROOT, "profiles")
+
+
+def workload_desc(w):
+    return (f"Wan2.1-1.3B attention layer: {w.chunk_tokens}-query chunk "
+            f"({w.chunk_frames} latent frames of {w.grid_h}x{w.grid_w}) x {w.slots}-key window "
+            f"({w.window_frames} frames), {w.heads} heads, d_c={w.d_c}, d_r={w.d_r}, "
+            f"batch {w.batch}; step = cache append + attention")
+
+
+def flops_per_step(w):
+    rows = w.batch * w.chunk_tokens * w.heads
+    attn = 2.0 * rows * w.slots * (w.d_c + w.d_r) + 2.0 * rows * w.slots * w.d_c
+    append = 2.0 * w.batch * w.chunk_tokens * w.hidden * (w.d_c + w.d_r)
+    return attn, append
+
+
+def append_bytes(w):
+    """Algorithmic HBM bytes of one append: x, both weights, gamma, positions in;
+    c and k rows out."""
+    n = w.batch * w.chunk_tokens
+    return (n * w.hidden * 2 + (w.d_c + w.d_r) * w.hidden * 2 + w.d_c * 2 + n * 3 * 4
+            + n * (w.d_c + w.d_r) * 2)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def kernel_source_hash(name):
+    src = os.path.join(ROOT, "paper_2605_30351_gb300", "csrc", name)
+    with open(src, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic(summary, kernel_src):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel source (else None)."""
+    p = os.path.join(PROFILES, summary)
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    if d.get("kernel_source_sha256_16") != kernel_source_hash(kernel_src):
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in getattr(self, "lines", []):
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for name, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        loaded = [s for s in sm if s > 0.5 * (mx or max(sm))] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------- CPU oracle
+def cpu_oracle_sample(w, budget_s=12.0, seed=5, tokens_per_batch=8):
+    """Time the float64 oracle (as it stands) on a bounded sample of the same
+    workload: the append of R tokens and the attention of those R tokens' 12
+    heads against the full window, R grown in batches until ~budget_s."""
+    from oracle import mla_oracle as O
+
+    spec = O.RopeSpec(w.rope_pairs, w.rope_axis_dims, w.rope_theta)
+    weights = synth.draw_layer_weights(w, seed)
+    f64 = lambda t: t.float().numpy().astype(np.float64)
+    wd, wk, g = f64(weights["w_dkv"]), f64(weights["w_kr"]), f64(weights["gamma_kv"])
+    c, k = synth.draw_cache_rows(w, w.slots, seed + 1, batch=1)
+    c, k = f64(c[0]), f64(k[0])
+    q_c, q_r = synth.draw_queries(w, w.chunk_tokens, seed + 2, batch=1)
+    x = synth.draw_tokens(w, w.chunk_tokens, seed + 3, batch=1)
+    pos = synth.grid_positions(w, w.window_frames - w.chunk_frames, w.chunk_frames, batch=1)
+    q_c, q_r, x, pos = f64(q_c[0]), f64(q_r[0]), f64(x), pos.numpy()
+    step = tokens_per_batch
+    done = 0
+    fl = 0.0
+    c0 = os.times()
+    t0 = time.perf_counter()
+    while done < w.chunk_tokens and time.perf_counter() - t0 < budget_s:
+        sl = slice(done, min(done + step, w.chunk_tokens))
+        n = sl.stop - sl.start
+        oc = O.OracleCache(1, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r)
+        oc.T = n  # one partial "frame" of n tokens: the same arithmetic per token
+        O.cache_append(oc, x[:, sl], wd, wk, pos[:, sl], 0, 1, gamma=g, eps=w.rms_eps, spec=spec)
+        O.latent_attention(q_c[sl], q_r[sl], pos[0, sl], c, k, w.head_dim, spec)
+        fl += 2.0 * n * w.hidden * (w.d_c + w.d_r)
+        fl += O.latent_attention_flops(n * w.heads, w.slots, w.d_c, w.d_r)
+        done += n
+    wall = time.perf_counter() - t0
+    c1 = os.times()
+    cpu = (c1.user - c0.user) + (c1.system - c0.system)
+    return {
+        "value": fl / wall / 1e12,
+        "unit": UNIT,
+        "cores": max(1, round(cpu / wall)),
+        "host_cores_available": len(os.sched_getaffinity(0)),
+        "kind": "oracle",
+        "sample": (f"float64 NumPy oracle: append + attention of {done} of {w.chunk_tokens} "
+                   f"query tokens (x{w.heads} heads) against the full {w.slots}-key window, "
+                   f"{wall:.1f} s"),
+        "seconds": wall,
+    }
+
+
+# ------------------------------------------------------------------ GPU arm
+class LayerSet:
+    """One layer's device state: weights, a full cache, the step's inputs."""
+
+    def __init__(self, w, seed, V):
+        self.w = w
+        wt = synth.draw_layer_weights(w, seed)
+        self.w_dkv = wt["w_dkv"].cuda()
+        self.w_kr = wt["w_kr"].cuda()
+        self.gamma = wt["gamma_kv"].cuda()
+        self.cache = V.LatentCache(V.make_config(w))
+        c, k = synth.draw_cache_rows(w, w.slots, seed + 1)
+        self.cache.c.copy_(c)
+        self.cache.kr.copy_(k)
+        self.cache.frames_written = w.window_frames
+        self.first = w.window_frames - w.chunk_frames
+        self.x = synth.draw_tokens(w, w.chunk_tokens, seed + 2).cuda()
+        self.pos = synth.grid_positions(w, self.first, w.chunk_frames).cuda()
+        q_c, q_r = synth.draw_queries(w, w.chunk_tokens, seed + 3)
+        self.q_c, self.q_r = q_c.cuda(), q_r.cuda()
+        self.o = torch.empty(w.batch, w.chunk_tokens, w.heads, w.d_c, dtype=torch.bfloat16,
+                             device="cuda")
+
+
+def run_ours(args, w, rank, world, local_rank):
+    from paper_2605_30351_gb300 import videomla as V
+
+    torch.cuda.set_device(local_rank)
+    V.load()
+    stream = torch.cuda.current_stream()
+    sets = [LayerSet(w, 1000 + 17 * i + 101 * rank, V) for i in range(N_SETS)]
+    attn_fl, app_fl = flops_per_step(w)
+
+    def step(s, ev=None):
+        V.mla_cache_append(s.cache, s.x, s.w_dkv, s.gamma, s.w_kr, s.pos, s.first,
+                           w.chunk_frames, stream)
+        if ev is not None:
+            ev[0].record(stream)
+        V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
+        if ev is not None:
+            ev[1].record(stream)
+
+    for i in range(args.warmup):
+        step(sets[i % N_SETS])
+    torch.cuda.synchronize()
+    assert V.mla_device_status(clear=True) == V.MLA_OK
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(sets[i % N_SETS], ev[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms_total = t_start.elapsed_time(t_end)
+    attn_ms = [a.elapsed_time(b) for a, b in ev]
+    ms_max = allreduce_max(ms_total, world)
+    status = V.mla_device_status(clear=True)
+    if status != V.MLA_OK:
+        raise RuntimeError(f"device status {status} after the timed region")
+
+    # end to end through the public API with pinned host buffers: H2D of the
+    # step's inputs, append + attention, D2H of the latent output
+    h_sets = []
+    for s in sets[:2]:
+        h_sets.append({"x": s.x.cpu().pin_memory(), "q_c": s.q_c.cpu().pin_memory(),
+                       "q_r": s.q_r.cpu().pin_memory(), "pos": s.pos.cpu().pin_memory(),
+                       "o": torch.empty_like(s.o, device="cpu").pin_memory()})
+    h2d = sum(h_sets[0][k].numel() * h_sets[0][k].element_size()
+              for k in ("x", "q_c", "q_r", "pos"))
+    d2h = h_sets[0]["o"].numel() * h_sets[0]["o"].element_size()
+    e2e_steps = max(3, args.steps // 4)
+
+    def e2e_step(i):
+        s, h = sets[i % 2], h_sets[i % 2]
+        s.x.copy_(h["x"], non_blocking=True)
+        s.q_c.copy_(h["q_c"], non_blocking=True)
+        s.q_r.copy_(h["q_r"], non_blocking=True)
+        s.pos.copy_(h["pos"], non_blocking=True)
+        step(s)
+        h["o"].copy_(s.o, non_blocking=True)
+
+    for i in range(2):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    barrier(world)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = allreduce_max(e0.elapsed_time(e1), world)
+
+    if rank != 0:
+        return None
+    peaks = load_peaks()
+    ms_step = ms_max / args.steps
+    attn_ms_mean = statistics.fmean(attn_ms)
+    achieved = attn_fl / (attn_ms_mean * 1e-3) / 1e12
+    app_ms = ms_step - attn_ms_mean
+    out = {
+        "metric": METRIC,
+        "value": world * (attn_fl + app_fl) / (ms_step * 1e-3) / 1e12,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded Gaussian activations, weights N(0,1/fan_in), "
+                "cache rows N(0,1)); no dataset or trained weights",
+        "config": {
+            "workload": workload_desc(w),
+            "queries": w.chunk_tokens * w.heads, "keys": w.slots, "heads": w.heads,
+            "d_c": w.d_c, "d_r": w.d_r, "hidden": w.hidden, "batch": w.batch,
+            "rope_pairs_thw": list(w.rope_pairs),
+            "l2": f"inputs larger than L2: {N_SETS} rotating layer sets "
+                  f"(~{N_SETS * 76} MB), one per step",
+            "parallelism": f"replicas x{world}",
+        },
+        "attention_ms": attn_ms_mean,
+        "append_ms_est": app_ms,
+        "roofline": {
+            "bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"],
+            "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"],
+            "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
+            "peak_source": f"{peaks['source']} bf16 dense (burst)",
+            "kernel": "mla_attn_tc_kernel<192,32>",
+            "algorithmic_flops_per_launch": attn_fl,
+            "traffic": profiled_traffic("attn_tc_wan_traffic.json", "attn_tc.cu"),
+        },
+        "roofline_append": {
+            "bound": "hbm", "kernel": "mla_append_tc_kernel<192,32>",
+            "algorithmic_bytes_per_launch": append_bytes(w),
+            "achieved": append_bytes(w) / max(app_ms, 1e-6) / 1e6,
+            "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": append_bytes(w) / max(app_ms, 1e-6) / 1e6 / peaks["hbm_gbs"],
+            "note": "append time = step time - attention event time (includes launch gaps)",
+        },
+        "e2e": {
+            "value": world * (attn_fl + app_fl) / (e2e_ms / e2e_steps * 1e-3) / 1e12,
+            "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": e2e_ms / e2e_steps, "steps": e2e_steps,
+        },
+        "clocks": clk.summary(),
+        "gpu_launches": 2 * args.steps,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_oracle_sample(w, budget_s=args.cpu_budget)
+    return out
+
+
+def run_reference(args, w, rank):
+    """The reference arm: the float64 oracle, as it stands, on the host cores."""
+    if rank != 0:
+        return None
+    # each step is a bounded sample; the whole run stays within a few minutes
+    budget = min(args.cpu_budget, 60.0 / max(1, args.steps + args.warmup))
+    tok = 8 if budget >= 1.0 else 1
+    for _ in range(args.warmup):
+        cpu_oracle_sample(w, budget_s=budget, tokens_per_batch=tok)
+    vals = [cpu_oracle_sample(w, budget_s=budget, tokens_per_batch=tok)
+            for _ in range(args.steps)]
+    v = statistics.fmean(x["value"] for x in vals)
+    cb = dict(vals[-1])
+    cb["value"] = v
+    return {
+        "impl": "reference",
+        "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": 0, "steps": args.steps,
+        "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_desc(w)},
+        "cpu_baseline": cb,
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+# -------------------------------------------------------------- distributed
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def allreduce_max(x, world):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="wan")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    w = synth.workload(args.workload)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and args.impl == "ours":
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    if args.impl == "reference":
+        out = run_reference(args, w, rank)
+    else:
+        out = run_ours(args, w, rank, world, local_rank)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+    if world > 1 and args.impl == "ours":
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
