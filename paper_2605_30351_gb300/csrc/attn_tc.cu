@@ -276,9 +276,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < kBN; ++c)
           if (c >= valid) sv[c] = -INFINITY;
       }
-      float mx = sv[0];
+      // row max as 8 independent chains + a 3-level tree (short dependency path)
+      float m8[8];
 #pragma unroll
-      for (int c = 1; c < kBN; ++c) mx = fmaxf(mx, sv[c]);
+      for (int i = 0; i < 8; ++i) m8[i] = sv[i];
+#pragma unroll
+      for (int c = 8; c < kBN; c += 8)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[c + i]);
+      const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                             fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       const float m_blk = mx * p.scale_log2;
       if (j == 0) {
         m_run = m_blk;
@@ -310,17 +317,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       const float neg_m = -m_run;
-      float l0 = 0.f, l1 = 0.f;
+      float l8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) l8[i] = 0.f;
       uint32_t pk[kBN / 2];
 #pragma unroll
       for (int i = 0; i < kBN / 2; ++i) {
         const float p0 = ex2_approx(fmaf(sv[2 * i], p.scale_log2, neg_m));
         const float p1 = ex2_approx(fmaf(sv[2 * i + 1], p.scale_log2, neg_m));
-        l0 += p0;
-        l1 += p1;
+        l8[(2 * i) & 7] += p0;
+        l8[(2 * i + 1) & 7] += p1;
         pk[i] = pack_bf16x2(p0, p1);
       }
-      l_run += l0 + l1;
+      l_run += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
 #pragma unroll
       for (int c = 0; c < kBN / 64; ++c)
         tmem_st32(t_s + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[c * 32]));

@@ -131,7 +131,7 @@ def grid_positions(w, first_frame, n_frames, batch=None):
     hh = np.tile(np.repeat(np.arange(w.grid_h), w.grid_w), n_frames)
     ww = np.tile(np.arange(w.grid_w), w.grid_h * n_frames)
     pos = np.stack([t, hh, ww], axis=-1).astype(np.int32)
-    return torch.from_numpy(np.array(np.broadcast_to(pos, (B,) + pos.shape)))
+    return torch.from_numpy(np.repeat(pos[None], B, axis=0))
 
 
 def draw_queries(w, n_tokens, seed, batch=None):
