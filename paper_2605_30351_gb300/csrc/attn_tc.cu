@@ -9,16 +9,29 @@
 //     O  += P . c                                  N = d_c (192), latent output
 // One CTA owns 128 rows (one TMEM lane each) and walks the window in blocks
 // of 128 keys:
-//   warp 0     TMA producer: q_c tile once, then [c | k] tiles into a ring of
-//              shared-memory stages (no multicast).
-//   warp 1     allocates TMEM; one lane issues every tcgen05.mma:
-//              S_j = Q K_j^T into TMEM buffer j%2 (SS form), then
-//              O += P_{j-1} V_{j-1} with P read from TMEM (TS form).
-//   warps 2-5  rotate q_r into the Q tile, then the online softmax: thread i
-//              owns row i, reads S_j from TMEM, writes P_j (bf16) over S_j's
-//              first half, rescales O in TMEM only when its running max grows
-//              by more than 2^8, and finally writes O / l as bf16.
-// The V operand is the first d_c columns of the same K tile read MN-major,
+//   warp 0     TMA producer: [c | k] tiles into a ring of shared-memory
+//              stages (c with 128-byte swizzle, k with 64-byte swizzle).
+//              CTAs run in pairs (a cluster of two consecutive row tiles of
+//              the same batch element): each CTA fetches half of every key
+//              tile from L2 and multicasts it into both CTAs' stage, halving
+//              the L2-to-SM traffic, which otherwise bounds the kernel.
+//   warp 1     allocates TMEM; one lane issues the score MMAs
+//              S_j = Q K_j^T with Q read from TMEM, so they read only the key
+//              tile from shared memory. S_{j+1} is issued as soon as the
+//              softmax has copied S_j into registers.
+//   warp 6     one lane issues O += P_j V_j with P read from TMEM. Two issuing
+//              threads keep the tensor pipe fed while either one waits on a
+//              barrier: the MMA queue is shallow, so a single issuer's
+//              bookkeeping between groups would leave the pipe idle.
+//   warps 2-5  load q_c, rotate q_r and store both into TMEM; then the online
+//              softmax: thread i owns row i, copies S_j out of TMEM (releasing
+//              it), writes P_j (bf16) once PV_{j-1} has read the previous P,
+//              rescales O in TMEM only when its running max grows by more
+//              than 2^8, and finally writes O / l as bf16.
+// TMEM columns: S [0,128) P [128,192) O [192,192+d_c) Q [192+d_c, +(d_c+d_r)/2).
+// When Q does not fit there (d_c = 256) it stays in shared memory (TMA-loaded
+// q_c plus the rotated q_r stored by the softmax warps) and QK reads it there.
+// The V operand is the first d_c columns of the same key tile read MN-major,
 // so the cache is never expanded into per-head keys or values.
 #include <cmath>
 
@@ -30,35 +43,41 @@ namespace {
 
 constexpr int kBM = 128;       // rows per CTA = TMEM lanes
 constexpr int kBN = 128;       // keys per block
-constexpr int kThreads = 192;  // 6 warps
+constexpr int kThreads = 224;  // 7 warps
 constexpr float kRescaleLog2 = 8.0f;
 
 template <int DC, int DR>
 struct AttnShape {
   static constexpr int DK = DC + DR;
-  static constexpr int kTileBytes = kBM * DK * 2;  // the Q tile and one KV stage (kBM == kBN)
-  static constexpr int kKrOff = DC * kBM * 2;      // byte offset of the d_r columns in a tile
+  static constexpr int kTileBytes = kBN * DK * 2;  // one key stage (and the smem Q tile)
+  static constexpr int kKrOff = DC * kBN * 2;      // byte offset of the d_r columns in a tile
+  static constexpr int kTmemS = 0;
+  static constexpr int kTmemP = kBN;               // bf16 P: two values per column
+  static constexpr int kTmemO = kBN + kBN / 2;
+  static constexpr int kTmemQ = kTmemO + DC;
+  static constexpr bool kQinTmem = kTmemQ + DK / 2 <= 512;
+  static constexpr int kQBytes = kQinTmem ? 0 : kBM * DK * 2;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmemCap = 232448;
-  static constexpr int kFit = (kSmemCap - 1024 - kBarBytes - kTileBytes) / kTileBytes;
+  static constexpr int kFit = (kSmemCap - 1024 - kBarBytes - kQBytes) / kTileBytes;
   static constexpr int kStages = kFit > 4 ? 4 : kFit;
-  static constexpr int kSmemBytes = 1024 + kTileBytes * (1 + kStages) + kBarBytes;
-  static constexpr int kTmemO = 2 * kBN;
+  static constexpr int kSmemBytes = 1024 + kQBytes + kTileBytes * kStages + kBarBytes;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kKrSw = DR == 32 ? kSw64 : kSw128;
-  static constexpr uint32_t kKrRow = DR * 2;     // bytes per row of the d_r block
+  static constexpr uint32_t kKrRow = DR * 2;      // bytes per row of the d_r block
   static constexpr uint32_t kKrSbo = 8 * kKrRow;  // one 8-row swizzle atom
   static constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
   static constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, DC, false, true);
-  static_assert(kBM == kBN, "the Q tile and a KV stage share one size");
+  static_assert(kBM == kBN, "the smem Q tile and a key stage share one layout");
   static_assert(DC % 64 == 0 && DC >= 64 && DC <= 256, "d_c: multiple of 64 up to 256");
   static_assert(DR == 32 || DR == 64, "d_r: 32 or 64");
-  static_assert(kTmemO + DC <= 512, "two S buffers plus O must fit in 512 TMEM columns");
-  static_assert(kStages >= 2, "at least two KV stages must fit in shared memory");
+  static_assert(kTmemO + DC <= 512, "S, P and O must fit in 512 TMEM columns");
+  static_assert(kStages >= 2, "at least two key stages must fit in shared memory");
   static_assert(kTileBytes % 1024 == 0 && kKrOff % 1024 == 0, "swizzle-atom alignment");
 };
 
 struct AttnKParams {
+  const __nv_bfloat16* q_c;
   const __nv_bfloat16* q_r;
   const int* q_pos;
   const float2* rope;
@@ -68,27 +87,30 @@ struct AttnKParams {
   int* status;
 };
 
-template <int DC, int DR>
+template <int DC, int DR, int CL>
 __global__ void __launch_bounds__(kThreads, 1)
     mla_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_qc,
                        const __grid_constant__ CUtensorMap tm_c,
                        const __grid_constant__ CUtensorMap tm_kr, const AttnKParams p) {
   using S = AttnShape<DC, DR>;
   constexpr int NST = S::kStages;
+  constexpr uint16_t kPair = static_cast<uint16_t>((1u << CL) - 1u);  // every CTA of the cluster
+  static_assert(CL == 1 || CL == 2, "clusters of one or two CTAs");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_smem_1024(smem_raw);
-  uint8_t* sQ = smem;
-  uint8_t* sKV = smem + S::kTileBytes;
+  uint8_t* sQ = smem;  // only when Q stays in shared memory
+  uint8_t* sKV = smem + S::kQBytes;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + NST * S::kTileBytes);
   uint64_t* q_tma_full = bars + 0;
-  uint64_t* q_rot_ready = bars + 1;
+  uint64_t* q_ready = bars + 1;
   uint64_t* kv_full = bars + 2;
   uint64_t* kv_empty = kv_full + NST;
   uint64_t* s_full = kv_empty + NST;
-  uint64_t* p_full = s_full + 2;
-  uint64_t* pv_done = p_full + 2;
-  uint64_t* mma_drain = pv_done + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_drain + 1);
+  uint64_t* s_free = s_full + 1;
+  uint64_t* p_full = s_free + 1;
+  uint64_t* pv_done = p_full + 1;
+  uint64_t* mma_drain = pv_done + 1;  // [2]: one per issuing thread
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_drain + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -100,17 +122,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_tma_full, 1);
-    mbar_init(q_rot_ready, kBM);
+    mbar_init(q_ready, kBM);
     for (int s = 0; s < NST; ++s) {
       mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&kv_empty[s], CL);  // released by the MMA of every CTA that reads it
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_full[i], 1);
-      mbar_init(&p_full[i], kBM);
-      mbar_init(&pv_done[i], 1);
-    }
-    mbar_init(mma_drain, 1);
+    mbar_init(s_full, 1);
+    mbar_init(s_free, kBM);
+    mbar_init(p_full, kBM);
+    mbar_init(pv_done, 1);
+    mbar_init(&mma_drain[0], 1);
+    mbar_init(&mma_drain[1], 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -122,54 +144,65 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // the peer's barriers must be initialised before any multicast lands
+  if constexpr (CL > 1) cluster_sync();
+  const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      tma_prefetch_desc(&tm_qc);
       tma_prefetch_desc(&tm_c);
       tma_prefetch_desc(&tm_kr);
-      mbar_arrive_expect_tx(q_tma_full, DC * kBM * 2);
-      for (int cb = 0; cb < DC / 64; ++cb)
-        tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, cb * 64, row0, b);
+      if constexpr (!S::kQinTmem) {
+        tma_prefetch_desc(&tm_qc);
+        mbar_arrive_expect_tx(q_tma_full, DC * kBM * 2);
+        for (int cb = 0; cb < DC / 64; ++cb)
+          tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, cb * 64, row0, b);
+      }
       int issued = 0;
       for (int j = 0; j < nblk; ++j) {
         const int st = j % NST;
         if (j >= NST && !mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, wc)) break;
         uint8_t* kv = sKV + st * S::kTileBytes;
         mbar_arrive_expect_tx(&kv_full[st], S::kTileBytes);
-        for (int cb = 0; cb < DC / 64; ++cb)
-          tma_load_3d(kv + cb * 16384, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
-        tma_load_3d(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b);
+        if constexpr (CL == 1) {
+          for (int cb = 0; cb < DC / 64; ++cb)
+            tma_load_3d(kv + cb * 16384, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
+          tma_load_3d(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b);
+        } else {
+          // each CTA fetches every other box once and multicasts it to both
+          for (int bx = crank; bx <= DC / 64; bx += CL) {
+            if (bx < DC / 64)
+              tma_load_3d_mc(kv + bx * 16384, &tm_c, &kv_full[st], bx * 64, j * kBN, b, kPair);
+            else
+              tma_load_3d_mc(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b, kPair);
+          }
+        }
         issued = j + 1;
       }
+      // every stage's last use must be released before the CTA may exit
+      for (int st = 0; st < NST && st < nblk && !*abort_flag; ++st)
+        mbar_wait(&kv_empty[st], (((nblk - st + NST - 1) / NST) - 1) & 1, wc);
       if (*abort_flag) {  // let every copy this CTA started land before exit
-        mbar_wait_drain(q_tma_full, 0, p.status);
+        if constexpr (!S::kQinTmem) mbar_wait_drain(q_tma_full, 0, p.status);
         for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
           mbar_wait_drain(&kv_full[u % NST], (u / NST) & 1, p.status);
       }
     }
+    __syncwarp();
   } else if (warp == 1) {
-    // ---------------------------------------------------------- MMA issuer
+    // ------------------------------------------------------ QK^T issuer
     if (lane == 0) {
-      bool ok = mbar_wait(q_tma_full, 0, wc) && mbar_wait(q_rot_ready, 0, wc);
+      bool ok = mbar_wait(q_ready, 0, wc);
+      if constexpr (!S::kQinTmem) ok = ok && mbar_wait(q_tma_full, 0, wc);
       tc_fence_after();
       const uint32_t qa = smem_u32(sQ);
-      auto issue_pv = [&](int i) -> bool {
-        if (!mbar_wait(&p_full[i & 1], (i >> 1) & 1, wc)) return false;
-        tc_fence_after();
-        const int st = i % NST;
-        const uint32_t va = smem_u32(sKV) + st * S::kTileBytes;
-        const uint32_t a_p = tmem + (i & 1) * kBN;  // bf16 P over S_i's first 64 columns
-#pragma unroll
-        for (int s = 0; s < kBN / 16; ++s)
-          umma_ts(tmem + S::kTmemO, a_p + s * 8, sdesc(va + s * 2048, 16384, 1024, kSw128),
-                  S::kIdescPV, (i > 0 || s > 0) ? 1u : 0u);
-        umma_commit(&kv_empty[st]);
-        umma_commit(&pv_done[i & 1]);
-        return true;
-      };
       for (int j = 0; ok && j < nblk; ++j) {
+        // S = Q K_j^T; S's previous contents (block j-1) must have been read
+        if (j >= 1 && !mbar_wait(s_free, (j - 1) & 1, wc)) {
+          ok = false;
+          break;
+        }
         const int st = j % NST;
         if (!mbar_wait(&kv_full[st], (j / NST) & 1, wc)) {
           ok = false;
@@ -177,25 +210,62 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const uint32_t ka = smem_u32(sKV) + st * S::kTileBytes;
-        const uint32_t d_s = tmem + (j & 1) * kBN;
 #pragma unroll
         for (int cb = 0; cb < DC / 64; ++cb)
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_ss(d_s, sdesc(qa + cb * 16384 + k * 32, 16, 1024, kSw128),
-                    sdesc(ka + cb * 16384 + k * 32, 16, 1024, kSw128), S::kIdescQK,
-                    (cb | k) != 0 ? 1u : 0u);
+          for (int k = 0; k < 4; ++k) {
+            const uint64_t bd = sdesc(ka + cb * 16384 + k * 32, 16, 1024, kSw128);
+            const uint32_t acc = (cb | k) != 0 ? 1u : 0u;
+            if constexpr (S::kQinTmem)
+              umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + (cb * 4 + k) * 8, bd, S::kIdescQK, acc);
+            else
+              umma_ss(tmem + S::kTmemS, sdesc(qa + cb * 16384 + k * 32, 16, 1024, kSw128), bd,
+                      S::kIdescQK, acc);
+          }
 #pragma unroll
-        for (int k = 0; k < DR / 16; ++k)
-          umma_ss(d_s, sdesc(qa + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw),
-                  sdesc(ka + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw), S::kIdescQK, 1u);
-        umma_commit(&s_full[j & 1]);
-        if (j > 0 && !issue_pv(j - 1)) ok = false;
+        for (int k = 0; k < DR / 16; ++k) {
+          const uint64_t bd = sdesc(ka + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw);
+          if constexpr (S::kQinTmem)
+            umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + DC / 2 + k * 8, bd, S::kIdescQK, 1u);
+          else
+            umma_ss(tmem + S::kTmemS, sdesc(qa + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw), bd,
+                    S::kIdescQK, 1u);
+        }
+        umma_commit(s_full);
       }
-      if (ok) ok = issue_pv(nblk - 1);
-      if (!ok) {  // wait for every MMA already issued before TMEM is freed
-        umma_commit(mma_drain);
-        mbar_wait_drain(mma_drain, 0, p.status);
+      if (!ok) {  // wait for every MMA this thread issued before TMEM is freed
+        umma_commit(&mma_drain[0]);
+        mbar_wait_drain(&mma_drain[0], 0, p.status);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 6) {
+    // --------------------------------------------------------- PV issuer
+    if (lane == 0) {
+      bool ok = true;
+      for (int i = 0; ok && i < nblk; ++i) {
+        // O += P_i V_i, V = the first d_c columns of block i's stage (MN-major)
+        if (!mbar_wait(p_full, i & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int st = i % NST;
+        const uint32_t va = smem_u32(sKV) + st * S::kTileBytes;
+#pragma unroll
+        for (int s = 0; s < kBN / 16; ++s)
+          umma_ts(tmem + S::kTmemO, tmem + S::kTmemP + s * 8,
+                  sdesc(va + s * 2048, 16384, 1024, kSw128), S::kIdescPV,
+                  (i > 0 || s > 0) ? 1u : 0u);
+        if constexpr (CL == 1)
+          umma_commit(&kv_empty[st]);
+        else
+          umma_commit_mc(&kv_empty[st], kPair);
+        umma_commit(pv_done);
+      }
+      if (!ok) {
+        umma_commit(&mma_drain[1]);
+        mbar_wait_drain(&mma_drain[1], 0, p.status);
       }
     }
     __syncwarp();
@@ -207,8 +277,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int grow = row0 + r;
     const bool row_ok = grow < p.rows;
 
-    // q_r -> RoPE3D(q_r) in bf16, written into the Q tile's d_r block using
-    // the same 16-byte-chunk swizzle the TMA would apply.
+    // Q: q_c as is, q_r rotated by the query position (RoPE3D), both bf16.
     {
       uint32_t w[DR / 2];
 #pragma unroll
@@ -241,32 +310,59 @@ __global__ void __launch_bounds__(kThreads, 1)
           w[i] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
         }
       }
-      uint8_t* krow = sQ + S::kKrOff + r * S::kKrRow;
+      if constexpr (S::kQinTmem) {
+        // TMEM holds the MMA's A operand row-major: column c = elements 2c, 2c+1
+        const uint4* qsrc = reinterpret_cast<const uint4*>(
+            p.q_c + (static_cast<size_t>(b) * p.rows + (row_ok ? grow : 0)) * DC);
 #pragma unroll
-      for (int c = 0; c < DR / 8; ++c) {
-        const int phys = DR == 32 ? (c ^ ((r >> 1) & 3)) : (c ^ (r & 7));
-        *reinterpret_cast<uint4*>(krow + phys * 16) =
-            make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+        for (int c = 0; c < DC / 64; ++c) {
+          uint32_t qw[32];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const uint4 v = row_ok ? __ldg(qsrc + c * 8 + i) : make_uint4(0u, 0u, 0u, 0u);
+            qw[4 * i + 0] = v.x;
+            qw[4 * i + 1] = v.y;
+            qw[4 * i + 2] = v.z;
+            qw[4 * i + 3] = v.w;
+          }
+          tmem_st32(tmem + t_lane + S::kTmemQ + c * 32, qw);
+        }
+#pragma unroll
+        for (int c = 0; c < DR / 32; ++c)
+          tmem_st16(tmem + t_lane + S::kTmemQ + DC / 2 + c * 16, w + c * 16);
+        tmem_wait_st();
+        tc_fence_before();
+      } else {
+        // the same 16-byte-chunk swizzle the TMA applies to the q_c part
+        uint8_t* krow = sQ + S::kKrOff + r * S::kKrRow;
+#pragma unroll
+        for (int c = 0; c < DR / 8; ++c) {
+          const int phys = DR == 32 ? (c ^ ((r >> 1) & 3)) : (c ^ (r & 7));
+          *reinterpret_cast<uint4*>(krow + phys * 16) =
+              make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+        }
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
-      mbar_arrive(q_rot_ready);
+      mbar_arrive(q_ready);
     }
 
     float m_run = -INFINITY;
     float l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
-      if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, wc)) {
+      if (!mbar_wait(s_full, j & 1, wc)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t t_s = tmem + t_lane + (j & 1) * kBN;
       uint32_t sr[kBN];
 #pragma unroll
       for (int c = 0; c < kBN / 32; ++c)
-        tmem_ld32(t_s + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
+        tmem_ld32(tmem + t_lane + S::kTmemS + c * 32,
+                  *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
       tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(s_free);  // S_j is in registers: the next block's scores may land
       float sv[kBN];
 #pragma unroll
       for (int c = 0; c < kBN; ++c) sv[c] = __uint_as_float(sr[c]);
@@ -287,35 +383,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                              fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       const float m_blk = mx * p.scale_log2;
+      // lazy rescale: keep the running max unless this block's max exceeds it
+      // by more than 2^8 (P <= 256 then, harmless in bf16 / fp32)
+      float alpha = 1.f;
+      bool need = false;
       if (j == 0) {
         m_run = m_blk;
-      } else {
-        const bool need = m_blk > m_run + kRescaleLog2;
-        if (__any_sync(0xffffffffu, need)) {
-          // O is only touched once PV_{j-1} has landed.
-          if (!mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, wc)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          float alpha = 1.f;
-          if (need) {
-            alpha = ex2_approx(m_run - m_blk);
-            m_run = m_blk;
-          }
-          l_run *= alpha;
-#pragma unroll 1
-          for (int c = 0; c < DC / 32; ++c) {
-            uint32_t ov[32];
-            tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * alpha);
-            tmem_st32(tmem + t_lane + S::kTmemO + c * 32, ov);
-          }
-          tmem_wait_st();
-        }
+      } else if (m_blk > m_run + kRescaleLog2) {
+        need = true;
+        alpha = ex2_approx(m_run - m_blk);
+        m_run = m_blk;
       }
+      l_run *= alpha;
+      // P_j in registers before waiting on PV_{j-1}: only the TMEM store
+      // below is serialised with the previous PV
       const float neg_m = -m_run;
       float l8[8];
 #pragma unroll
@@ -330,15 +411,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         pk[i] = pack_bf16x2(p0, p1);
       }
       l_run += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
+      if (j > 0) {
+        // PV_{j-1} must have read P (and finished with O) before P_j is
+        // written or O is rescaled
+        if (!mbar_wait(pv_done, (j - 1) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, need)) {
+#pragma unroll 1
+          for (int c = 0; c < DC / 32; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * alpha);
+            tmem_st32(tmem + t_lane + S::kTmemO + c * 32, ov);
+          }
+          tmem_wait_st();
+        }
+      }
 #pragma unroll
       for (int c = 0; c < kBN / 64; ++c)
-        tmem_st32(t_s + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[c * 32]));
+        tmem_st32(tmem + t_lane + S::kTmemP + c * 32,
+                  *reinterpret_cast<uint32_t(*)[32]>(&pk[c * 32]));
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&p_full[j & 1]);
+      mbar_arrive(p_full);
     }
 
-    if (ok && mbar_wait(&pv_done[(nblk - 1) & 1], ((nblk - 1) >> 1) & 1, wc)) {
+    if (ok && mbar_wait(pv_done, (nblk - 1) & 1, wc)) {
       tc_fence_after();
       const float inv_l = 1.f / l_run;
       uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC);
@@ -367,9 +470,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, S::kTmemCols);
   }
+  // neither CTA leaves while the other may still write into its shared memory
+  if constexpr (CL > 1) cluster_sync();
 }
 
-template <int DC, int DR>
+template <int DC, int DR, int CL>
 int launch_tc(const AttnArgs& a) {
   using S = AttnShape<DC, DR>;
   CUtensorMap tm_qc, tm_c, tm_kr;
@@ -382,7 +487,7 @@ int launch_tc(const AttnArgs& a) {
                           kBN,
                           DR == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
-  auto kern = mla_attn_tc_kernel<DC, DR>;
+  auto kern = mla_attn_tc_kernel<DC, DR, CL>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
   if (e != cudaSuccess) {
@@ -390,6 +495,7 @@ int launch_tc(const AttnArgs& a) {
     return MLA_ERR_CUDA;
   }
   AttnKParams kp;
+  kp.q_c = static_cast<const __nv_bfloat16*>(a.q_c);
   kp.q_r = static_cast<const __nv_bfloat16*>(a.q_r);
   kp.q_pos = a.q_pos;
   kp.rope = reinterpret_cast<const float2*>(a.rope);
@@ -402,9 +508,21 @@ int launch_tc(const AttnArgs& a) {
   kp.pairs_h = a.pairs_h;
   kp.scale_log2 = a.scale_log2;
   kp.status = a.status;
-  const dim3 grid((a.rows + kBM - 1) / kBM, a.batch);
-  kern<<<grid, kThreads, S::kSmemBytes, a.stream>>>(tm_qc, tm_c, tm_kr, kp);
-  e = cudaGetLastError();
+  const int tiles = (a.rows + kBM - 1) / kBM;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((tiles + CL - 1) / CL * CL, a.batch, 1);  // pairs stay within a batch row
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = S::kSmemBytes;
+  cfg.stream = a.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, tm_qc, tm_c, tm_kr, kp);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return MLA_ERR_CUDA;
@@ -412,22 +530,29 @@ int launch_tc(const AttnArgs& a) {
   return MLA_OK;
 }
 
+// Pairs of CTAs share every key tile through TMA multicast; a single row tile
+// per batch element runs alone.
+template <int DC, int DR>
+int launch_tc_pick(const AttnArgs& a) {
+  return (a.rows + kBM - 1) / kBM >= 2 ? launch_tc<DC, DR, 2>(a) : launch_tc<DC, DR, 1>(a);
+}
+
 }  // namespace
 
 int launch_attention_tc(const AttnArgs& a) {
   if (a.d_r == 32) {
     switch (a.d_c) {
-      case 64: return launch_tc<64, 32>(a);
-      case 128: return launch_tc<128, 32>(a);
-      case 192: return launch_tc<192, 32>(a);
-      case 256: return launch_tc<256, 32>(a);
+      case 64: return launch_tc_pick<64, 32>(a);
+      case 128: return launch_tc_pick<128, 32>(a);
+      case 192: return launch_tc_pick<192, 32>(a);
+      case 256: return launch_tc_pick<256, 32>(a);
       default: break;
     }
   } else if (a.d_r == 64) {
     switch (a.d_c) {
-      case 64: return launch_tc<64, 64>(a);
-      case 128: return launch_tc<128, 64>(a);
-      case 192: return launch_tc<192, 64>(a);
+      case 64: return launch_tc_pick<64, 64>(a);
+      case 128: return launch_tc_pick<128, 64>(a);
+      case 192: return launch_tc_pick<192, 64>(a);
       default: break;
     }
   }
