@@ -34,6 +34,9 @@ struct AppendShape {
   static constexpr int kStages = kFit > 6 ? 6 : kFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
   static constexpr uint32_t kTmemCols = N <= 256 ? 256 : 512;
+  // output staging row: N bf16 plus 16 bytes, so rows start on different banks
+  static constexpr int kOutStride = N * 2 + 16;
+  static_assert(kBM * kOutStride + kBM * 8 <= kStages * kStageBytes, "staging fits in the ring");
   static_assert(DC % 32 == 0 && DR % 32 == 0 && DC <= 256 && DR <= 64, "shape");
   static_assert(N <= 512, "accumulator must fit in TMEM");
   static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
@@ -152,7 +155,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_row = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int n = row0 + r;
     const bool row_ok = n < p.n_tok;
-    if (mbar_wait(acc_full, 0, wc) && !*abort_flag) {
+    const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
+    // The finished bf16 rows are staged in shared memory (the stage ring is
+    // free once the accumulator is complete) and then written out by all 128
+    // threads together, so that consecutive threads store consecutive 16-byte
+    // pieces of a row instead of each thread writing its own row.
+    uint8_t* stage_out = smem;                                   // [128][kOutStride]
+    long long* slot_of = reinterpret_cast<long long*>(smem + kBM * S::kOutStride);  // [128]
+    if (have_acc) {
       tc_fence_after();
       // pass 1: mean square of c over d_c (fp32)
       float ss = 0.f;
@@ -169,30 +179,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
       const long long f = p.first_frame + n / p.T;
-      const long long slot = (f % p.W) * p.T + n % p.T;
-      uint4* cdst = reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC);
-      // pass 2: gamma * c / rms -> bf16 -> ring slot
+      slot_of[r] = row_ok ? (f % p.W) * p.T + n % p.T : -1;
+      uint8_t* srow = stage_out + r * S::kOutStride;
+      // pass 2: gamma * c / rms -> bf16
 #pragma unroll 1
       for (int cb = 0; cb < DC / 32; ++cb) {
         uint32_t v[32];
         tmem_ld32(t_row + cb * 32, v);
         tmem_wait_ld();
+        uint32_t gw[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          uint4 g4 = make_uint4(0x3f803f80u, 0x3f803f80u, 0x3f803f80u, 0x3f803f80u);  // ones
+          if (p.gamma) g4 = __ldg(reinterpret_cast<const uint4*>(p.gamma + cb * 32) + i);
+          gw[4 * i] = g4.x; gw[4 * i + 1] = g4.y; gw[4 * i + 2] = g4.z; gw[4 * i + 3] = g4.w;
+        }
         uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float g0 = 1.f, g1 = 1.f;
-          if (p.gamma) {
-            g0 = __bfloat162float(p.gamma[cb * 32 + 2 * i]);
-            g1 = __bfloat162float(p.gamma[cb * 32 + 2 * i + 1]);
-          }
-          pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]) * inv * g0,
-                              __uint_as_float(v[2 * i + 1]) * inv * g1);
-        }
-        if (row_ok) {
+        for (int i = 0; i < 16; ++i)
+          pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]) * inv * bf16_lo(gw[i]),
+                              __uint_as_float(v[2 * i + 1]) * inv * bf16_hi(gw[i]));
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            cdst[cb * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-        }
+        for (int i = 0; i < 4; ++i)
+          *reinterpret_cast<uint4*>(srow + cb * 64 + i * 16) =
+              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
       // positional key: RoPE3D at the token's (t, h, w)
       int pa[3] = {0, 0, 0};
@@ -208,7 +218,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             pa[a] = 0;
           }
       }
-      uint4* kdst = reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR);
 #pragma unroll 1
       for (int cb = 0; cb < DR / 32; ++cb) {
         uint32_t v[32];
@@ -223,11 +232,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
           pk[i] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
         }
-        if (row_ok) {
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            kdst[cb * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-        }
+        for (int i = 0; i < 4; ++i)
+          *reinterpret_cast<uint4*>(srow + DC * 2 + cb * 64 + i * 16) =
+              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+      }
+    }
+    // the four epilogue warps only
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (have_acc) {
+      constexpr int kChunks = S::N * 2 / 16;  // 16-byte pieces per output row
+      constexpr int kChunksC = DC * 2 / 16;
+      for (int q = r; q < kBM * kChunks; q += kBM) {
+        const int row = q / kChunks, ch = q % kChunks;
+        const long long slot = slot_of[row];
+        if (slot < 0) continue;
+        const uint4 v = *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
+        if (ch < kChunksC)
+          *reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC + ch * 8) = v;
+        else
+          *reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR +
+                                    (ch - kChunksC) * 8) = v;
       }
     }
   }
