@@ -302,7 +302,7 @@ def run_ours(args, w, rank, world, local_rank):
     app_ms = statistics.fmean(app_ms_l)
     out = {
         "metric": METRIC,
-        "value": world * (attn_fl + app_fl) / (ms_step * 1e-3) / 1e12,
+        "value": whole_job_throughput(attn_fl + app_fl, ms_step, world),
         "unit": UNIT,
         "n_gpus": world,
         "steps": args.steps,
@@ -343,7 +343,7 @@ def run_ours(args, w, rank, world, local_rank):
             "note": "CUDA events around each append launch (mean over the timed steps)",
         },
         "e2e": {
-            "value": world * (attn_fl + app_fl) / (e2e_ms / e2e_steps * 1e-3) / 1e12,
+            "value": whole_job_throughput(attn_fl + app_fl, e2e_ms / e2e_steps, world),
             "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": e2e_ms / e2e_steps, "steps": e2e_steps,
         },
@@ -387,11 +387,19 @@ def barrier(world):
 
 
 def allreduce_max(x, world):
+    """Max of a per-rank scalar over all ranks (timing: the slowest replica)."""
     if world == 1:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if torch.distributed.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_throughput(flop_per_step_per_rank, ms_per_step_max, world):
+    """Replicas: every rank does the same work; the job rate is the sum of the
+    ranks' work over the slowest rank's time, in TFLOP/s."""
+    return world * flop_per_step_per_rank / (ms_per_step_max * 1e-3) / 1e12
 
 
 def main():
