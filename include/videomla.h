@@ -44,7 +44,7 @@ extern "C" {
  *                  sqrt(head_dim) (Eq. score)
  *  d_c             width of the shared KV latent c^KV (192)   (Eq. ckv)
  *  d_r             width of the shared positional key k^R (32) (Eq. krope)
- *  d_q             width of the query latent (768); informational here
+ *  d_q             width of the query latent c^Q (768), used by the query prologue
  *  rope_pairs_*    complex pairs per axis; 2*(t+h+w) must equal d_r (App. D.3)
  *  rope_dim_*      band width D_a of each axis: pair i of axis a rotates with
  *                  theta^(-2i/D_a), i.e. the highest-frequency bands of the
@@ -159,6 +159,55 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv,
 int mla_attention_forward(const mla_cache* cache, const void* q_c,
                           const void* q_r, const int* q_pos, int Nq,
                           void* o_lat, void* stream);
+
+/*
+ * Load-time weight absorption (App. E, Eqs. absorb-q and absorb-v), computed
+ * on the device with fp32 accumulation and rounded once to bf16:
+ *   w_qcat bf16 [H*(d_c+d_r)][d_q]: rows (h, c), c < d_c, hold
+ *          A_h[:, c] * gamma_q = sum_e W_up,h^Q[e][:] W_up,h^K[e][c] * gamma_q,
+ *          rows H*d_c + (h, j) hold W_R,h^Q[j][:] * gamma_q (Eq. qrope);
+ *   w_b    bf16 [hidden][H*d_c]: B_h = W_O,h W_up,h^V side by side.
+ * Inputs (bf16): w_uq [H][d_nope][d_q], w_uk [H][d_nope][d_c],
+ * w_qr [H][d_r][d_q], gamma_q [d_q] or NULL (ones), w_uv [H][d_h][d_c],
+ * w_o [hidden][H*d_h]; d_nope = head_dim - d_r. Asynchronous on `stream`.
+ */
+int mla_absorb_weights(const mla_config* cfg, const void* w_uq, const void* w_uk,
+                       const void* w_qr, const void* gamma_q, const void* w_uv,
+                       const void* w_o, void* w_qcat, void* w_b, void* stream);
+
+/* Bytes of caller-owned device workspace mla_query_prologue needs for Nq
+ * query tokens per batch element (0 on a bad config). */
+unsigned long long mla_query_workspace_bytes(const mla_config* cfg, int Nq);
+
+/*
+ * Query path of a chunk (Eqs. cq, qnope, qrope; App. D.2 RMSNorm; App. E):
+ *     c~        = W_dn^Q x                       (bf16 in the workspace)
+ *     [q_c|q_r] = [W_qc ; W_qr] diag(gamma_q) c~ / rms(c~)
+ * The RMSNorm statistics come from the fp32 accumulator of the first GEMM;
+ * the per-row scale is applied in the second GEMM's epilogue (it commutes
+ * with the linear map). Outputs are exactly mla_attention_forward's inputs:
+ *  x       bf16 [batch][Nq][hidden]
+ *  w_dq    bf16 [d_q][hidden]
+ *  w_qcat  bf16 [H*(d_c+d_r)][d_q] from mla_absorb_weights
+ *  workspace  device memory of at least mla_query_workspace_bytes(cfg, Nq)
+ *             bytes, 16-byte aligned, owned by the caller; its contents are
+ *             scratch between the two GEMMs of this call
+ *  q_c     bf16 [batch][Nq][H][d_c];  q_r bf16 [batch][Nq][H][d_r] (unrotated)
+ * MLA_ERR_UNSUPPORTED unless d_q and hidden are multiples of 64.
+ */
+int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq,
+                       const void* w_qcat, int Nq, void* workspace,
+                       unsigned long long workspace_bytes, void* q_c, void* q_r,
+                       void* stream);
+
+/*
+ * Output projection of the latent attention output (Eq. absorb-v):
+ *     y = sum_h B_h o_lat,h = o_lat W_B^T
+ *  o_lat bf16 [batch][Nq][H][d_c], w_b bf16 [hidden][H*d_c],
+ *  y bf16 [batch][Nq][hidden]. MLA_ERR_UNSUPPORTED unless H*d_c % 64 == 0.
+ */
+int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* w_b, int Nq,
+                          void* y, void* stream);
 
 /* Human-readable name of a status code. */
 const char* mla_status_string(int status);

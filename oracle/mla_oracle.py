@@ -60,6 +60,8 @@ __all__ = [
     "reference_attention",
     "absorb_query",
     "absorb_output",
+    "absorbed_query_matrices",
+    "absorbed_output_matrices",
     "per_head_output_from_latent",
     "cache_scalars_per_token",
     "dense_scalars_per_token",
@@ -287,6 +289,20 @@ def absorb_query(c_q, w_uq, w_uk):
     """q_c,h = A_h^T c^Q with A_h = (W_up,h^Q)^T W_up,h^K  (Eq. absorb-q)."""
     A = np.einsum("heq,hec->hqc", w_uq, w_uk)       # [H, d_q, d_c]
     return np.einsum("hqc,nq->nhc", A, np.asarray(c_q, dtype=np.float64))
+
+
+def absorbed_query_matrices(w_uq, w_uk):
+    """A_h = (W_up,h^Q)^T W_up,h^K in R^{d_q x d_c}, stacked over heads (App. E)."""
+    return np.einsum("heq,hec->hqc", np.asarray(w_uq, dtype=np.float64),
+                     np.asarray(w_uk, dtype=np.float64))
+
+
+def absorbed_output_matrices(w_uv, w_o):
+    """B_h = W_O,h W_up,h^V in R^{d x d_c}, stacked over heads (App. E)."""
+    w_uv = np.asarray(w_uv, dtype=np.float64)
+    w_o = np.asarray(w_o, dtype=np.float64)
+    H, d_v, _ = w_uv.shape
+    return np.stack([w_o[:, h * d_v:(h + 1) * d_v] @ w_uv[h] for h in range(H)])
 
 
 def per_head_output_from_latent(o_lat, w_uv):

@@ -260,6 +260,97 @@ int mla_attention_forward(const mla_cache* cache, const void* q_c, const void* q
   return (c.flags & MLA_FLAG_SIMT) ? launch_attention_simt(a) : launch_attention_tc(a);
 }
 
+int mla_absorb_weights(const mla_config* cfg, const void* w_uq, const void* w_uk, const void* w_qr,
+                       const void* gamma_q, const void* w_uv, const void* w_o, void* w_qcat,
+                       void* w_b, void* stream) {
+  const int rc = check_config(cfg);
+  if (rc != MLA_OK) return rc;
+  if (!w_uq || !w_uk || !w_qr || !w_uv || !w_o || !w_qcat || !w_b) return MLA_ERR_ARG;
+  if (cfg->head_dim <= cfg->d_r || cfg->d_q <= 0) return MLA_ERR_ARG;
+  AbsorbArgs a;
+  a.w_uq = w_uq;
+  a.w_uk = w_uk;
+  a.w_qr = w_qr;
+  a.gamma_q = gamma_q;
+  a.w_uv = w_uv;
+  a.w_o = w_o;
+  a.w_qcat = w_qcat;
+  a.w_b = w_b;
+  a.hidden = cfg->hidden;
+  a.heads = cfg->heads;
+  a.head_dim = cfg->head_dim;
+  a.d_c = cfg->d_c;
+  a.d_r = cfg->d_r;
+  a.d_q = cfg->d_q;
+  a.stream = static_cast<cudaStream_t>(stream);
+  return launch_absorb(a);
+}
+
+unsigned long long mla_query_workspace_bytes(const mla_config* cfg, int Nq) {
+  if (check_config(cfg) != MLA_OK || Nq < 1 || cfg->d_q <= 0) return 0;
+  const unsigned long long rows = static_cast<unsigned long long>(cfg->batch) * Nq;
+  const unsigned long long ct = (rows * cfg->d_q * 2 + 255) / 256 * 256;
+  return ct + static_cast<unsigned long long>((cfg->d_q + 255) / 256) * rows * 4;
+}
+
+int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq, const void* w_qcat,
+                       int Nq, void* workspace, unsigned long long workspace_bytes, void* q_c,
+                       void* q_r, void* stream) {
+  const int rc = check_config(cfg);
+  if (rc != MLA_OK) return rc;
+  if (!x || !w_dq || !w_qcat || !workspace || !q_c || !q_r || Nq < 1) return MLA_ERR_ARG;
+  if (!aligned16(x) || !aligned16(w_dq) || !aligned16(w_qcat) || !aligned16(workspace) ||
+      !aligned16(q_c) || !aligned16(q_r))
+    return MLA_ERR_ARG;
+  if (cfg->d_q <= 0 || cfg->d_q % 64 != 0 || cfg->hidden % 64 != 0) return MLA_ERR_UNSUPPORTED;
+  if (workspace_bytes < mla_query_workspace_bytes(cfg, Nq)) return MLA_ERR_ARG;
+  const long long rows = static_cast<long long>(cfg->batch) * Nq;
+  if (rows > (1ll << 30)) return MLA_ERR_ARG;
+  QueryArgs a;
+  a.x = x;
+  a.w_dq = w_dq;
+  a.w_qcat = w_qcat;
+  a.c_tilde = workspace;
+  a.sq = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                  (rows * cfg->d_q * 2 + 255) / 256 * 256);
+  a.q_c = q_c;
+  a.q_r = q_r;
+  a.rows = static_cast<int>(rows);
+  a.hidden = cfg->hidden;
+  a.heads = cfg->heads;
+  a.d_c = cfg->d_c;
+  a.d_r = cfg->d_r;
+  a.d_q = cfg->d_q;
+  a.eps = cfg->rms_eps;
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return launch_query_prologue(a);
+}
+
+int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* w_b, int Nq,
+                          void* y, void* stream) {
+  const int rc = check_config(cfg);
+  if (rc != MLA_OK) return rc;
+  if (!o_lat || !w_b || !y || Nq < 1) return MLA_ERR_ARG;
+  if (!aligned16(o_lat) || !aligned16(w_b) || !aligned16(y)) return MLA_ERR_ARG;
+  if ((cfg->heads * cfg->d_c) % 64 != 0) return MLA_ERR_UNSUPPORTED;
+  const long long rows = static_cast<long long>(cfg->batch) * Nq;
+  if (rows > (1ll << 30)) return MLA_ERR_ARG;
+  OutProjArgs a;
+  a.o_lat = o_lat;
+  a.w_b = w_b;
+  a.y = y;
+  a.rows = static_cast<int>(rows);
+  a.hidden = cfg->hidden;
+  a.heads = cfg->heads;
+  a.d_c = cfg->d_c;
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return launch_output_projection(a);
+}
+
 const char* mla_status_string(int status) {
   switch (status) {
     case MLA_OK: return "ok";

@@ -1,0 +1,336 @@
+// Dense bf16 GEMMs around the attention (tcgen05, TMEM accumulator, TMA):
+// the query prologue (Eqs. cq, qnope, qrope with App. E's absorbed weights)
+// and the output projection (Eq. absorb-v). C[M x N] = A[M x K] B[N x K]^T,
+// both operands K-major, fp32 accumulation, one 128 x BN tile per CTA:
+//   warp 0     TMA producer (A [128 x 64], B [BN x 64] per stage, SW128)
+//   warp 1     TMEM allocation; one lane issues tcgen05.mma (N = BN)
+//   warps 2-5  epilogue, thread i = row i: TMEM -> registers -> bf16 staged
+//              in shared memory, then stored by all 128 threads together.
+// Epilogues:
+//   kStore      plain bf16 C
+//   kStoreSq    bf16 C plus, per row, the sum of squares of this tile's fp32
+//               columns (RMSNorm's statistics, App. D.2)
+//   kRowScale   every row scaled by 1/sqrt(mean of the squares + eps) before
+//               rounding, columns [0, split) to C and [split, N) to C2.
+// RMSNorm's per-row scale commutes with the following linear map, so the
+// query latent is normalised in the next GEMM's epilogue: q = (W diag(gamma))
+// c~ / rms(c~), with gamma folded into W when the weights are absorbed.
+#include <cmath>
+
+#include "internal.h"
+#include "ptx_sm103.cuh"
+
+namespace vmla {
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+
+template <int BN>
+struct GemmShape {
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kFit = (232448 - 1024 - kBarBytes) / kStageBytes;
+  static constexpr int kStages = kFit > 6 ? 6 : kFit;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
+  static constexpr int kOutStride = BN * 2 + 16;  // staged bf16 row + 16 bytes (bank spread)
+  static constexpr uint32_t kTmemCols = BN <= 128 ? 128 : 256;
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN, false, false);
+  static_assert(BN % 32 == 0 && BN <= 256, "tile width");
+  static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
+  static_assert(kBM * kOutStride <= kStages * kStageBytes, "staging fits in the ring");
+};
+
+struct GemmKParams {
+  __nv_bfloat16* c;       // [M][ldc] (columns [0, split) when kRowScale)
+  __nv_bfloat16* c2;      // kRowScale: [M][ld2] for columns [split, N)
+  float* sq;              // kStoreSq: out [n_tiles][M]; kRowScale: in [sq_tiles][M]
+  int M, N, K, ldc, ld2, split, sq_tiles;
+  float sq_dim, eps;
+  int* status;
+};
+
+enum { kStore = 0, kStoreSq = 1, kRowScale = 2 };
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_gemm_tc_kernel(const __grid_constant__ CUtensorMap tm_a,
+                       const __grid_constant__ CUtensorMap tm_b, const GemmKParams p) {
+  using S = GemmShape<BN>;
+  constexpr int NST = S::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align_smem_1024(smem_raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NST * S::kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + NST;
+  uint64_t* acc_full = bars + 2 * NST;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * kBM;
+  const int n0 = blockIdx.y * BN;
+  const int k_blocks = p.K / kBK;
+  const WaitCtx wc{abort_flag, p.status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(acc_full, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, S::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_a);
+      tma_prefetch_desc(&tm_b);
+      int issued = 0;
+      for (int kb = 0; kb < k_blocks; ++kb) {
+        const int st = kb % NST;
+        if (kb >= NST && !mbar_wait(&empty[st], ((kb / NST) - 1) & 1, wc)) break;
+        uint8_t* a = smem + st * S::kStageBytes;
+        mbar_arrive_expect_tx(&full[st], S::kStageBytes);
+        tma_load_2d(a, &tm_a, &full[st], kb * kBK, m0);
+        tma_load_2d(a + S::kABytes, &tm_b, &full[st], kb * kBK, n0);
+        issued = kb + 1;
+      }
+      if (*abort_flag)
+        for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
+          mbar_wait_drain(&full[u % NST], (u / NST) & 1, p.status);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = true;
+      for (int kb = 0; kb < k_blocks; ++kb) {
+        const int st = kb % NST;
+        if (!mbar_wait(&full[st], (kb / NST) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t aa = smem_u32(smem + st * S::kStageBytes);
+        const uint32_t ba = aa + S::kABytes;
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          umma_ss(tmem, sdesc(aa + k * 32, 16, 1024, kSw128), sdesc(ba + k * 32, 16, 1024, kSw128),
+                  S::kIdesc, (kb | k) != 0 ? 1u : 0u);
+        umma_commit(&empty[st]);
+      }
+      umma_commit(acc_full);
+      if (!ok) mbar_wait_drain(acc_full, 0, p.status);
+    }
+    __syncwarp();
+  } else {
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t t_row = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    const int m = m0 + r;
+    const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
+    uint8_t* stage_out = smem;  // [128][kOutStride]
+    const int n_valid = min(BN, p.N - n0);
+    if (have_acc) {
+      tc_fence_after();
+      float scale = 1.f;
+      if constexpr (EPI == kRowScale) {
+        float ss = 0.f;
+        if (m < p.M)
+          for (int t = 0; t < p.sq_tiles; ++t) ss += p.sq[static_cast<size_t>(t) * p.M + m];
+        scale = rsqrtf(ss / p.sq_dim + p.eps);
+      }
+      float ss_own = 0.f;
+      uint8_t* srow = stage_out + r * S::kOutStride;
+#pragma unroll 1
+      for (int cb = 0; cb < BN / 32; ++cb) {
+        uint32_t v[32];
+        tmem_ld32(t_row + cb * 32, v);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float a0 = __uint_as_float(v[2 * i]), a1 = __uint_as_float(v[2 * i + 1]);
+          if constexpr (EPI == kStoreSq) {
+            const int col = cb * 32 + 2 * i;
+            if (col < n_valid) ss_own = fmaf(a0, a0, ss_own);
+            if (col + 1 < n_valid) ss_own = fmaf(a1, a1, ss_own);
+          }
+          pk[i] = pack_bf16x2(a0 * scale, a1 * scale);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          *reinterpret_cast<uint4*>(srow + cb * 64 + i * 16) =
+              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+      }
+      if constexpr (EPI == kStoreSq)
+        if (m < p.M) p.sq[static_cast<size_t>(blockIdx.y) * p.M + m] = ss_own;
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
+    if (have_acc) {
+      const int chunks = n_valid / 8;  // 16-byte pieces per row (N is a multiple of 8)
+      for (int q = r; q < kBM * chunks; q += kBM) {
+        const int row = q / chunks, ch = q % chunks;
+        const int mm = m0 + row;
+        if (mm >= p.M) continue;
+        const uint4 v = *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
+        const int col = n0 + ch * 8;
+        if (EPI == kRowScale && col >= p.split)
+          *reinterpret_cast<uint4*>(p.c2 + static_cast<size_t>(mm) * p.ld2 + (col - p.split)) = v;
+        else
+          *reinterpret_cast<uint4*>(p.c + static_cast<size_t>(mm) * p.ldc + col) = v;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, S::kTmemCols);
+  }
+}
+
+template <int BN, int EPI>
+int launch_gemm(const void* a, const void* b, int M, int N, int K, GemmKParams kp,
+                cudaStream_t stream) {
+  using S = GemmShape<BN>;
+  if (K % kBK != 0 || N % 8 != 0) return MLA_ERR_UNSUPPORTED;
+  CUtensorMap tm_a, tm_b;
+  if (!encode_map_2d_bf16(&tm_a, a, K, M, K * 2ull, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_2d_bf16(&tm_b, b, K, N, K * 2ull, kBK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+    return MLA_ERR_CUDA;
+  auto kern = mla_gemm_tc_kernel<BN, EPI>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  kp.M = M;
+  kp.N = N;
+  kp.K = K;
+  const dim3 grid((M + kBM - 1) / kBM, (N + BN - 1) / BN);
+  kern<<<grid, kThreads, S::kSmemBytes, stream>>>(tm_a, tm_b, kp);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  return MLA_OK;
+}
+
+// ---- load-time weight absorption (App. E), fp32 accumulation, bf16 out ----
+// w_qcat row (h, c) for c < d_c: sum_e W_uq[h][e][q] W_uk[h][e][c] * gamma_q[q]
+//        row H*d_c + (h, j):     W_qr[h][j][q] * gamma_q[q]
+__global__ void absorb_query_kernel(const __nv_bfloat16* __restrict__ w_uq,
+                                    const __nv_bfloat16* __restrict__ w_uk,
+                                    const __nv_bfloat16* __restrict__ w_qr,
+                                    const __nv_bfloat16* __restrict__ gamma_q,
+                                    __nv_bfloat16* __restrict__ w_qcat, int H, int dn, int dc,
+                                    int dr, int dq) {
+  const long long idx = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+  const long long rows = static_cast<long long>(H) * (dc + dr);
+  if (idx >= rows * dq) return;
+  const int row = static_cast<int>(idx / dq), q = static_cast<int>(idx % dq);
+  const float g = gamma_q ? __bfloat162float(gamma_q[q]) : 1.f;
+  float acc = 0.f;
+  if (row < H * dc) {
+    const int h = row / dc, c = row % dc;
+    for (int e = 0; e < dn; ++e)
+      acc = fmaf(__bfloat162float(w_uq[(static_cast<size_t>(h) * dn + e) * dq + q]),
+                 __bfloat162float(w_uk[(static_cast<size_t>(h) * dn + e) * dc + c]), acc);
+  } else {
+    const int rr = row - H * dc;  // (h, j) -> w_qr[h][j][q]
+    acc = __bfloat162float(w_qr[static_cast<size_t>(rr) * dq + q]);
+  }
+  w_qcat[idx] = __float2bfloat16_rn(acc * g);
+}
+
+// w_b[i][(h, c)] = sum_v W_o[i][h*dh + v] W_uv[h][v][c]
+__global__ void absorb_output_kernel(const __nv_bfloat16* __restrict__ w_uv,
+                                     const __nv_bfloat16* __restrict__ w_o,
+                                     __nv_bfloat16* __restrict__ w_b, int d, int H, int dh,
+                                     int dc) {
+  const long long idx = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+  if (idx >= static_cast<long long>(d) * H * dc) return;
+  const int i = static_cast<int>(idx / (H * dc));
+  const int hc = static_cast<int>(idx % (H * dc));
+  const int h = hc / dc, c = hc % dc;
+  float acc = 0.f;
+  for (int v = 0; v < dh; ++v)
+    acc = fmaf(__bfloat162float(w_o[static_cast<size_t>(i) * H * dh + h * dh + v]),
+               __bfloat162float(w_uv[(static_cast<size_t>(h) * dh + v) * dc + c]), acc);
+  w_b[idx] = __float2bfloat16_rn(acc);
+}
+
+}  // namespace
+
+int launch_absorb(const AbsorbArgs& a) {
+  const long long nq = static_cast<long long>(a.heads) * (a.d_c + a.d_r) * a.d_q;
+  const long long nb = static_cast<long long>(a.hidden) * a.heads * a.d_c;
+  absorb_query_kernel<<<static_cast<unsigned>((nq + 255) / 256), 256, 0, a.stream>>>(
+      static_cast<const __nv_bfloat16*>(a.w_uq), static_cast<const __nv_bfloat16*>(a.w_uk),
+      static_cast<const __nv_bfloat16*>(a.w_qr), static_cast<const __nv_bfloat16*>(a.gamma_q),
+      static_cast<__nv_bfloat16*>(a.w_qcat), a.heads, a.head_dim - a.d_r, a.d_c, a.d_r, a.d_q);
+  absorb_output_kernel<<<static_cast<unsigned>((nb + 255) / 256), 256, 0, a.stream>>>(
+      static_cast<const __nv_bfloat16*>(a.w_uv), static_cast<const __nv_bfloat16*>(a.w_o),
+      static_cast<__nv_bfloat16*>(a.w_b), a.hidden, a.heads, a.head_dim, a.d_c);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  return MLA_OK;
+}
+
+int launch_query_prologue(const QueryArgs& a) {
+  const int M = a.rows;  // batch * Nq tokens
+  const int sq_tiles = (a.d_q + 255) / 256;
+  // c~ = x W_dq^T (bf16) with per-row partial sums of squares
+  GemmKParams k1 = {};
+  k1.c = static_cast<__nv_bfloat16*>(a.c_tilde);
+  k1.ldc = a.d_q;
+  k1.sq = a.sq;
+  k1.status = a.status;
+  int rc = launch_gemm<256, kStoreSq>(a.x, a.w_dq, M, a.d_q, a.hidden, k1, a.stream);
+  if (rc != MLA_OK) return rc;
+  // [q_c | q_r] = (c~ / rms(c~)) [W_qc ; W_qr]^T with gamma folded into the weights
+  GemmKParams k2 = {};
+  k2.c = static_cast<__nv_bfloat16*>(a.q_c);
+  k2.ldc = a.heads * a.d_c;
+  k2.c2 = static_cast<__nv_bfloat16*>(a.q_r);
+  k2.ld2 = a.heads * a.d_r;
+  k2.split = a.heads * a.d_c;
+  k2.sq = a.sq;
+  k2.sq_tiles = sq_tiles;
+  k2.sq_dim = static_cast<float>(a.d_q);
+  k2.eps = a.eps;
+  k2.status = a.status;
+  return launch_gemm<256, kRowScale>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r), a.d_q,
+                                     k2, a.stream);
+}
+
+int launch_output_projection(const OutProjArgs& a) {
+  GemmKParams k = {};
+  k.c = static_cast<__nv_bfloat16*>(a.y);
+  k.ldc = a.hidden;
+  k.status = a.status;
+  return launch_gemm<256, kStore>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
+                                  a.stream);
+}
+
+}  // namespace vmla

@@ -45,11 +45,53 @@ struct AppendArgs {
   cudaStream_t stream;
 };
 
+// Load-time absorption of the per-head up-projections (App. E).
+struct AbsorbArgs {
+  const void* w_uq;     // bf16 [H][d_nope][d_q]
+  const void* w_uk;     // bf16 [H][d_nope][d_c]
+  const void* w_qr;     // bf16 [H][d_r][d_q]
+  const void* gamma_q;  // bf16 [d_q] or nullptr
+  const void* w_uv;     // bf16 [H][d_h][d_c]
+  const void* w_o;      // bf16 [hidden][H*d_h]
+  void* w_qcat;         // bf16 [H*(d_c+d_r)][d_q]
+  void* w_b;            // bf16 [hidden][H*d_c]
+  int hidden, heads, head_dim, d_c, d_r, d_q;
+  cudaStream_t stream;
+};
+
+// Query prologue: x -> c~ (+ row statistics) -> [q_c | q_r].
+struct QueryArgs {
+  const void* x;        // bf16 [rows][hidden]
+  const void* w_dq;     // bf16 [d_q][hidden]
+  const void* w_qcat;   // bf16 [H*(d_c+d_r)][d_q]
+  void* c_tilde;        // workspace bf16 [rows][d_q]
+  float* sq;            // workspace fp32 [ceil(d_q/256)][rows]
+  void* q_c;            // bf16 [rows][H*d_c]
+  void* q_r;            // bf16 [rows][H*d_r]
+  int rows, hidden, heads, d_c, d_r, d_q;
+  float eps;
+  int* status;
+  cudaStream_t stream;
+};
+
+// Output projection y = o_lat W_B^T.
+struct OutProjArgs {
+  const void* o_lat;    // bf16 [rows][H*d_c]
+  const void* w_b;      // bf16 [hidden][H*d_c]
+  void* y;              // bf16 [rows][hidden]
+  int rows, hidden, heads, d_c;
+  int* status;
+  cudaStream_t stream;
+};
+
 // Each launcher returns MLA_OK, MLA_ERR_UNSUPPORTED or MLA_ERR_CUDA.
 int launch_attention_tc(const AttnArgs& a);
 int launch_attention_simt(const AttnArgs& a);
 int launch_append_tc(const AppendArgs& a);
 int launch_append_simt(const AppendArgs& a);
+int launch_absorb(const AbsorbArgs& a);
+int launch_query_prologue(const QueryArgs& a);
+int launch_output_projection(const OutProjArgs& a);
 
 // Shared by the launchers: cuTensorMapEncodeTiled fetched from the driver.
 // Encodes a rank-3 bf16 tiled map over [d2][d1][d0] (d0 contiguous) with

@@ -28,6 +28,8 @@ MLA_FLAG_SIMT = 2
 # Every symbol include/videomla.h declares.
 EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
+           "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
+           "mla_output_projection",
            "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
 
 
@@ -84,9 +86,16 @@ def load():
     lib.mla_last_cuda_error.argtypes = []
     lib.mla_device_status.argtypes = [P(I), I]
     lib.mla_version.argtypes = []
+    lib.mla_absorb_weights.argtypes = [P(mla_config), VP, VP, VP, VP, VP, VP, VP, VP, VP]
+    lib.mla_query_workspace_bytes.argtypes = [P(mla_config), I]
+    lib.mla_query_workspace_bytes.restype = ctypes.c_ulonglong
+    lib.mla_query_prologue.argtypes = [P(mla_config), VP, VP, VP, I, VP, ctypes.c_ulonglong, VP,
+                                       VP, VP]
+    lib.mla_output_projection.argtypes = [P(mla_config), VP, VP, I, VP, VP]
     for name in ("mla_rope_table_fill", "mla_config_check", "mla_cache_reset", "mla_cache_append",
                  "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
-                 "mla_version"):
+                 "mla_version", "mla_absorb_weights", "mla_query_prologue",
+                 "mla_output_projection"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -209,6 +218,61 @@ def mla_attention_forward(cache, q_c, q_r, q_pos, o_lat, stream=None):
     _check("mla_attention_forward",
            load().mla_attention_forward(ctypes.byref(cache.struct), *args, int(Nq), out,
                                         _stream_ptr(stream)))
+
+
+def absorbed_weight_shapes(cfg):
+    """Shapes of (w_qcat, w_b) that mla_absorb_weights writes."""
+    return ((cfg.heads * (cfg.d_c + cfg.d_r), cfg.d_q), (cfg.hidden, cfg.heads * cfg.d_c))
+
+
+def mla_absorb_weights(cfg, w_uq, w_uk, w_qr, gamma_q, w_uv, w_o, stream=None):
+    """Absorbed query and output weights (App. E) as new bf16 CUDA tensors."""
+    H, dc, dr, dq, d, dh = cfg.heads, cfg.d_c, cfg.d_r, cfg.d_q, cfg.hidden, cfg.head_dim
+    dn = dh - dr
+    bf = torch.bfloat16
+    args = (
+        _dev(w_uq, bf, (H, dn, dq), "w_uq"), _dev(w_uk, bf, (H, dn, dc), "w_uk"),
+        _dev(w_qr, bf, (H, dr, dq), "w_qr"),
+        None if gamma_q is None else _dev(gamma_q, bf, (dq,), "gamma_q"),
+        _dev(w_uv, bf, (H, dh, dc), "w_uv"), _dev(w_o, bf, (d, H * dh), "w_o"),
+    )
+    sq, sb = absorbed_weight_shapes(cfg)
+    w_qcat = torch.empty(sq, dtype=bf, device=w_uq.device)
+    w_b = torch.empty(sb, dtype=bf, device=w_uq.device)
+    _check("mla_absorb_weights",
+           load().mla_absorb_weights(ctypes.byref(cfg), *args, ctypes.c_void_p(w_qcat.data_ptr()),
+                                     ctypes.c_void_p(w_b.data_ptr()), _stream_ptr(stream)))
+    return w_qcat, w_b
+
+
+def mla_query_workspace_bytes(cfg, Nq):
+    return int(load().mla_query_workspace_bytes(ctypes.byref(cfg), int(Nq)))
+
+
+def mla_query_prologue(cfg, x, w_dq, w_qcat, workspace, q_c, q_r, stream=None):
+    Nq = x.shape[1]
+    bf = torch.bfloat16
+    H, dc, dr, dq, d = cfg.heads, cfg.d_c, cfg.d_r, cfg.d_q, cfg.hidden
+    if not (isinstance(workspace, torch.Tensor) and workspace.is_cuda and workspace.is_contiguous()):
+        raise TypeError("workspace must be a contiguous CUDA tensor")
+    _check("mla_query_prologue",
+           load().mla_query_prologue(
+               ctypes.byref(cfg), _dev(x, bf, (cfg.batch, Nq, d), "x"),
+               _dev(w_dq, bf, (dq, d), "w_dq"), _dev(w_qcat, bf, (H * (dc + dr), dq), "w_qcat"),
+               int(Nq), ctypes.c_void_p(workspace.data_ptr()),
+               workspace.numel() * workspace.element_size(),
+               _dev(q_c, bf, (cfg.batch, Nq, H, dc), "q_c"),
+               _dev(q_r, bf, (cfg.batch, Nq, H, dr), "q_r"), _stream_ptr(stream)))
+
+
+def mla_output_projection(cfg, o_lat, w_b, y, stream=None):
+    Nq = o_lat.shape[1]
+    bf = torch.bfloat16
+    _check("mla_output_projection",
+           load().mla_output_projection(
+               ctypes.byref(cfg), _dev(o_lat, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "o_lat"),
+               _dev(w_b, bf, (cfg.hidden, cfg.heads * cfg.d_c), "w_b"), int(Nq),
+               _dev(y, bf, (cfg.batch, Nq, cfg.hidden), "y"), _stream_ptr(stream)))
 
 
 def mla_device_status(clear=True):

@@ -380,3 +380,22 @@ def test_brute_force_loops():
             z = sum(e)
             ref = [sum(e[j] * vals[j][i] for j in range(len(e))) / z for i in range(dh)]
             np.testing.assert_allclose(o[n, h], ref, rtol=1e-11, atol=1e-12)
+
+
+def test_absorbed_matrices_apply_like_the_absorbed_maps():
+    """A_h and B_h applied as matrices equal absorb_query / absorb_output, and
+    B_h o_lat,h equals W_O,h (W_up,h^V o_lat,h) -- the two groupings of Eq. absorb-v."""
+    rng = _rng(12)
+    H, dn, dq, dc, dh, d = 3, 4, 6, 5, 7, 9
+    w_uq, w_uk = rng.standard_normal((H, dn, dq)), rng.standard_normal((H, dn, dc))
+    w_uv, w_o = rng.standard_normal((H, dh, dc)), rng.standard_normal((d, H * dh))
+    c_q = rng.standard_normal((4, dq))
+    A = O.absorbed_query_matrices(w_uq, w_uk)
+    np.testing.assert_allclose(np.einsum("hqc,nq->nhc", A, c_q), O.absorb_query(c_q, w_uq, w_uk),
+                               rtol=1e-12, atol=1e-12)
+    o_lat = rng.standard_normal((4, H, dc))
+    B = O.absorbed_output_matrices(w_uv, w_o)
+    y = np.einsum("hdc,nhc->nd", B, o_lat)
+    o_h = O.per_head_output_from_latent(o_lat, w_uv)
+    np.testing.assert_allclose(y, o_h.reshape(4, -1) @ w_o.T, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(O.absorb_output(o_lat, w_uv, w_o), y, rtol=1e-12, atol=1e-12)
