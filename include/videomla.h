@@ -31,6 +31,10 @@ extern "C" {
 #define MLA_ERR_RANGE (-3)       /* frame count or position outside the window/table */
 #define MLA_ERR_CUDA (-4)        /* launch or runtime error (see mla_last_cuda_error) */
 #define MLA_ERR_TIMEOUT (-5)     /* a bounded device-side wait ran out */
+#define MLA_ERR_TOO_LARGE (-6)   /* request does not fit the library's fixed scratch */
+
+/* Size of the fixed device scratch used by mla_query_prologue_noalloc. */
+#define MLA_NOALLOC_SCRATCH_BYTES (8u * 1024u * 1024u)
 
 /* cfg.flags */
 #define MLA_FLAG_NO_RMSNORM 1u   /* store c^KV = W_dkv x without RMSNorm (App. D.2 off) */
@@ -199,6 +203,31 @@ int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq,
                        const void* w_qcat, int Nq, void* workspace,
                        unsigned long long workspace_bytes, void* q_c, void* q_r,
                        void* stream);
+
+/*
+ * mla_query_prologue without a caller workspace: the same computation and
+ * outputs, but the intermediate c~ and its row statistics live in a fixed
+ * array inside the library. The paper has no counterpart of this entry point;
+ * it exists for callers that cannot allocate device memory at the point of
+ * the call, e.g. code running inside another framework's memory pool or a
+ * real-time loop where any cudaMalloc/cudaFree would stall or be forbidden.
+ *  - Nothing is allocated: no cudaMalloc, cudaFree or allocating library call.
+ *  - The array holds MLA_NOALLOC_SCRATCH_BYTES bytes on every GPU that loads
+ *    the library, for the life of the process. Requests whose
+ *    mla_query_workspace_bytes(cfg, Nq) exceed it return MLA_ERR_TOO_LARGE
+ *    before anything is enqueued (the Wan-1.3B chunk of 4680 tokens at batch 1
+ *    needs about 7.2 MB and fits).
+ *  - The first call on each device looks up the array's device address with
+ *    cudaGetSymbolAddress; make that first call before any stream capture.
+ *  - All calls share the one array, and it keeps the previous call's
+ *    contents (nothing in it needs to start at zero: every call overwrites
+ *    what it reads). Calls whose work overlaps on the GPU, e.g. on two
+ *    streams at once, race on it; serialise them.
+ * Arguments and outputs as for mla_query_prologue.
+ */
+int mla_query_prologue_noalloc(const mla_config* cfg, const void* x, const void* w_dq,
+                               const void* w_qcat, int Nq, void* q_c, void* q_r,
+                               void* stream);
 
 /*
  * Output projection of the latent attention output (Eq. absorb-v):

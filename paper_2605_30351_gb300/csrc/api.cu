@@ -328,6 +328,44 @@ int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq, c
   return launch_query_prologue(a);
 }
 
+int mla_query_prologue_noalloc(const mla_config* cfg, const void* x, const void* w_dq,
+                               const void* w_qcat, int Nq, void* q_c, void* q_r, void* stream) {
+  const int rc = check_config(cfg);
+  if (rc != MLA_OK) return rc;
+  if (!x || !w_dq || !w_qcat || !q_c || !q_r || Nq < 1) return MLA_ERR_ARG;
+  if (!aligned16(x) || !aligned16(w_dq) || !aligned16(w_qcat) || !aligned16(q_c) ||
+      !aligned16(q_r))
+    return MLA_ERR_ARG;
+  if (cfg->d_q <= 0 || cfg->d_q % 64 != 0 || cfg->hidden % 64 != 0) return MLA_ERR_UNSUPPORTED;
+  const unsigned long long need = mla_query_workspace_bytes(cfg, Nq);
+  if (need == 0) return MLA_ERR_ARG;
+  if (need > MLA_NOALLOC_SCRATCH_BYTES) return MLA_ERR_TOO_LARGE;
+  void* scratch = nullptr;
+  const int sr = query_scratch_address(&scratch);
+  if (sr != MLA_OK) return sr;
+  const long long rows = static_cast<long long>(cfg->batch) * Nq;
+  QueryArgs a;
+  a.x = x;
+  a.w_dq = w_dq;
+  a.w_qcat = w_qcat;
+  a.c_tilde = scratch;
+  a.sq = reinterpret_cast<float*>(static_cast<char*>(scratch) +
+                                  (rows * cfg->d_q * 2 + 255) / 256 * 256);
+  a.q_c = q_c;
+  a.q_r = q_r;
+  a.rows = static_cast<int>(rows);
+  a.hidden = cfg->hidden;
+  a.heads = cfg->heads;
+  a.d_c = cfg->d_c;
+  a.d_r = cfg->d_r;
+  a.d_q = cfg->d_q;
+  a.eps = cfg->rms_eps;
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return launch_query_prologue(a);
+}
+
 int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* w_b, int Nq,
                           void* y, void* stream) {
   const int rc = check_config(cfg);
@@ -359,6 +397,7 @@ const char* mla_status_string(int status) {
     case MLA_ERR_RANGE: return "frame count or position out of range";
     case MLA_ERR_CUDA: return "CUDA error";
     case MLA_ERR_TIMEOUT: return "device wait timed out";
+    case MLA_ERR_TOO_LARGE: return "request exceeds the fixed no-allocation scratch";
     default: return "unknown status";
   }
 }

@@ -16,6 +16,7 @@
 // query latent is normalised in the next GEMM's epilogue: q = (W diag(gamma))
 // c~ / rms(c~), with gamma folded into W when the weights are absorbed.
 #include <cmath>
+#include <mutex>
 
 #include "internal.h"
 #include "ptx_sm103.cuh"
@@ -322,6 +323,41 @@ int launch_query_prologue(const QueryArgs& a) {
   k2.status = a.status;
   return launch_gemm<256, kRowScale>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r), a.d_q,
                                      k2, a.stream);
+}
+
+// ---- fixed scratch for mla_query_prologue_noalloc ----
+// The library's only device memory of its own: a file-scope array every GPU
+// that loads the library holds until the process exits. Host code must not
+// pass the symbol itself to a kernel (on the host it names a host-side
+// stand-in); query_scratch_address() looks up the device address instead.
+namespace {
+static __device__ __align__(256) unsigned char g_query_scratch[MLA_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxScratchDevices = 64;
+void* g_scratch_addr[kMaxScratchDevices] = {nullptr};
+std::mutex g_scratch_mu;
+}  // namespace
+
+int query_scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kMaxScratchDevices) return MLA_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {  // once per device, with that device current
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_query_scratch);
+    if (e != cudaSuccess || !p) {
+      set_last_cuda_error(e);
+      return MLA_ERR_CUDA;
+    }
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return MLA_OK;
 }
 
 int launch_output_projection(const OutProjArgs& a) {

@@ -92,6 +92,8 @@ int launch_append_simt(const AppendArgs& a);
 int launch_absorb(const AbsorbArgs& a);
 int launch_query_prologue(const QueryArgs& a);
 int launch_output_projection(const OutProjArgs& a);
+// Device address of the fixed no-allocation scratch on the current device.
+int query_scratch_address(void** out);
 
 // Shared by the launchers: cuTensorMapEncodeTiled fetched from the driver.
 // Encodes a rank-3 bf16 tiled map over [d2][d1][d0] (d0 contiguous) with

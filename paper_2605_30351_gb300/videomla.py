@@ -21,6 +21,8 @@ MLA_ERR_UNSUPPORTED = -2
 MLA_ERR_RANGE = -3
 MLA_ERR_CUDA = -4
 MLA_ERR_TIMEOUT = -5
+MLA_ERR_TOO_LARGE = -6
+MLA_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 MLA_FLAG_NO_RMSNORM = 1
 MLA_FLAG_SIMT = 2
@@ -29,7 +31,7 @@ MLA_FLAG_SIMT = 2
 EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
-           "mla_output_projection",
+           "mla_query_prologue_noalloc", "mla_output_projection",
            "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
 
 
@@ -92,10 +94,11 @@ def load():
     lib.mla_query_prologue.argtypes = [P(mla_config), VP, VP, VP, I, VP, ctypes.c_ulonglong, VP,
                                        VP, VP]
     lib.mla_output_projection.argtypes = [P(mla_config), VP, VP, I, VP, VP]
+    lib.mla_query_prologue_noalloc.argtypes = [P(mla_config), VP, VP, VP, I, VP, VP, VP]
     for name in ("mla_rope_table_fill", "mla_config_check", "mla_cache_reset", "mla_cache_append",
                  "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
-                 "mla_output_projection"):
+                 "mla_query_prologue_noalloc", "mla_output_projection"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -262,6 +265,21 @@ def mla_query_prologue(cfg, x, w_dq, w_qcat, workspace, q_c, q_r, stream=None):
                int(Nq), ctypes.c_void_p(workspace.data_ptr()),
                workspace.numel() * workspace.element_size(),
                _dev(q_c, bf, (cfg.batch, Nq, H, dc), "q_c"),
+               _dev(q_r, bf, (cfg.batch, Nq, H, dr), "q_r"), _stream_ptr(stream)))
+
+
+def mla_query_prologue_noalloc(cfg, x, w_dq, w_qcat, q_c, q_r, stream=None):
+    """The query prologue for callers that cannot allocate device memory: the
+    intermediate buffer is the library's fixed scratch (see the C header for
+    its size limit and the rule that overlapping calls race on it)."""
+    Nq = x.shape[1]
+    bf = torch.bfloat16
+    H, dc, dr, dq, d = cfg.heads, cfg.d_c, cfg.d_r, cfg.d_q, cfg.hidden
+    _check("mla_query_prologue_noalloc",
+           load().mla_query_prologue_noalloc(
+               ctypes.byref(cfg), _dev(x, bf, (cfg.batch, Nq, d), "x"),
+               _dev(w_dq, bf, (dq, d), "w_dq"), _dev(w_qcat, bf, (H * (dc + dr), dq), "w_qcat"),
+               int(Nq), _dev(q_c, bf, (cfg.batch, Nq, H, dc), "q_c"),
                _dev(q_r, bf, (cfg.batch, Nq, H, dr), "q_r"), _stream_ptr(stream)))
 
 
