@@ -34,13 +34,15 @@ PROFILES = os.path.join(ROOT, "profiles")
 
 
 def workload_desc(w):
+    layers = f"{w.layers} layers (distinct weights and caches), " if w.layers > 1 else ""
+    pos = f"; latent frames up to {w.last_frame - 1} (ring wrapped)" if w.last_frame > w.window_frames else ""
     return (f"Wan2.1-1.3B attention layer: {w.chunk_tokens}-query chunk "
             f"({w.chunk_frames} latent frames of {w.grid_h}x{w.grid_w}) x {w.slots}-key window "
             f"({w.window_frames} frames), {w.heads} heads, d_c={w.d_c}, d_r={w.d_r}, "
-            f"batch {w.batch}; step = cache append + attention")
+            f"batch {w.batch}; step = {layers}cache append + attention{pos}")
 
 
-def flops_per_step(w):
+def flops_per_layer(w):
     rows = w.batch * w.chunk_tokens * w.heads
     attn = 2.0 * rows * w.slots * (w.d_c + w.d_r) + 2.0 * rows * w.slots * w.d_c
     append = 2.0 * w.batch * w.chunk_tokens * w.hidden * (w.d_c + w.d_r)
@@ -48,8 +50,8 @@ def flops_per_step(w):
 
 
 def append_bytes(w):
-    """Algorithmic HBM bytes of one append: x, both weights, gamma, positions in;
-    c and k rows out."""
+    """Algorithmic HBM bytes of one append (one layer): x, both weights, gamma,
+    positions in; c and k rows out."""
     n = w.batch * w.chunk_tokens
     return (n * w.hidden * 2 + (w.d_c + w.d_r) * w.hidden * 2 + w.d_c * 2 + n * 3 * 4
             + n * (w.d_c + w.d_r) * 2)
@@ -203,8 +205,8 @@ class LayerSet:
         c, k = synth.draw_cache_rows(w, w.slots, seed + 1)
         self.cache.c.copy_(c)
         self.cache.kr.copy_(k)
-        self.cache.frames_written = w.window_frames
-        self.first = w.window_frames - w.chunk_frames
+        self.cache.frames_written = w.last_frame
+        self.first = w.last_frame - w.chunk_frames
         self.x = synth.draw_tokens(w, w.chunk_tokens, seed + 2).cuda()
         self.pos = synth.grid_positions(w, self.first, w.chunk_frames).cuda()
         q_c, q_r = synth.draw_queries(w, w.chunk_tokens, seed + 3)
@@ -219,10 +221,13 @@ def run_ours(args, w, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     V.load()
     stream = torch.cuda.current_stream()
-    sets = [LayerSet(w, 1000 + 17 * i + 101 * rank, V) for i in range(N_SETS)]
-    attn_fl, app_fl = flops_per_step(w)
+    # one set per layer of a step, or N_SETS rotating sets for a one-layer step
+    n_sets = max(w.layers, N_SETS)
+    sets = [LayerSet(w, 1000 + 17 * i + 101 * rank, V) for i in range(n_sets)]
+    attn_l, app_l = flops_per_layer(w)
+    attn_fl, app_fl = attn_l * w.layers, app_l * w.layers
 
-    def step(s, ev=None):
+    def layer(s, ev=None):
         if ev is not None:
             ev[0].record(stream)
         V.mla_cache_append(s.cache, s.x, s.w_dkv, s.gamma, s.w_kr, s.pos, s.first,
@@ -233,13 +238,17 @@ def run_ours(args, w, rank, world, local_rank):
         if ev is not None:
             ev[2].record(stream)
 
+    def step(i, evs=None):
+        for L in range(w.layers):
+            layer(sets[(i * w.layers + L) % n_sets], None if evs is None else evs[L])
+
     for i in range(args.warmup):
-        step(sets[i % N_SETS])
+        step(i)
     torch.cuda.synchronize()
     assert V.mla_device_status(clear=True) == V.MLA_OK
 
-    ev = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(3))
-          for _ in range(args.steps)]
+    ev = [[tuple(torch.cuda.Event(enable_timing=True) for _ in range(3))
+           for _ in range(w.layers)] for _ in range(args.steps)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -247,13 +256,13 @@ def run_ours(args, w, rank, world, local_rank):
     with ClockSampler(local_rank) as clk:
         t_start.record(stream)
         for i in range(args.steps):
-            step(sets[i % N_SETS], ev[i])
+            step(i, ev[i])
         t_end.record(stream)
         torch.cuda.synchronize()
     barrier(world)
     ms_total = t_start.elapsed_time(t_end)
-    app_ms_l = [e[0].elapsed_time(e[1]) for e in ev]
-    attn_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    app_ms_l = [e[0].elapsed_time(e[1]) for es in ev for e in es]
+    attn_ms = [e[1].elapsed_time(e[2]) for es in ev for e in es]
     ms_max = allreduce_max(ms_total, world)
     status = V.mla_device_status(clear=True)
     if status != V.MLA_OK:
@@ -262,23 +271,28 @@ def run_ours(args, w, rank, world, local_rank):
     # end to end through the public API with pinned host buffers: H2D of the
     # step's inputs, append + attention, D2H of the latent output
     h_sets = []
-    for s in sets[:2]:
+    n_e2e = max(2, w.layers)
+    for s in sets[:n_e2e]:
         h_sets.append({"x": s.x.cpu().pin_memory(), "q_c": s.q_c.cpu().pin_memory(),
                        "q_r": s.q_r.cpu().pin_memory(), "pos": s.pos.cpu().pin_memory(),
                        "o": torch.empty_like(s.o, device="cpu").pin_memory()})
-    h2d = sum(h_sets[0][k].numel() * h_sets[0][k].element_size()
-              for k in ("x", "q_c", "q_r", "pos"))
-    d2h = h_sets[0]["o"].numel() * h_sets[0]["o"].element_size()
+    h2d = w.layers * sum(h_sets[0][k].numel() * h_sets[0][k].element_size()
+                         for k in ("x", "q_c", "q_r", "pos"))
+    d2h = w.layers * h_sets[0]["o"].numel() * h_sets[0]["o"].element_size()
     e2e_steps = max(3, args.steps // 4)
+    if w.layers > 1:
+        e2e_steps = max(3, min(e2e_steps, 10))
 
     def e2e_step(i):
-        s, h = sets[i % 2], h_sets[i % 2]
-        s.x.copy_(h["x"], non_blocking=True)
-        s.q_c.copy_(h["q_c"], non_blocking=True)
-        s.q_r.copy_(h["q_r"], non_blocking=True)
-        s.pos.copy_(h["pos"], non_blocking=True)
-        step(s)
-        h["o"].copy_(s.o, non_blocking=True)
+        for L in range(w.layers):
+            j = (i * w.layers + L) % n_e2e
+            s, h = sets[j], h_sets[j]
+            s.x.copy_(h["x"], non_blocking=True)
+            s.q_c.copy_(h["q_c"], non_blocking=True)
+            s.q_r.copy_(h["q_r"], non_blocking=True)
+            s.pos.copy_(h["pos"], non_blocking=True)
+            layer(s)
+            h["o"].copy_(s.o, non_blocking=True)
 
     for i in range(2):
         e2e_step(i)
@@ -298,7 +312,7 @@ def run_ours(args, w, rank, world, local_rank):
     peaks = load_peaks()
     ms_step = ms_max / args.steps
     attn_ms_mean = statistics.fmean(attn_ms)
-    achieved = attn_fl / (attn_ms_mean * 1e-3) / 1e12
+    achieved = attn_l / (attn_ms_mean * 1e-3) / 1e12
     app_ms = statistics.fmean(app_ms_l)
     out = {
         "metric": METRIC,
@@ -323,6 +337,7 @@ def run_ours(args, w, rank, world, local_rank):
                   f"(~{N_SETS * 76} MB), one per step",
             "parallelism": f"replicas x{world}",
         },
+        "ms_per_layer": ms_step / w.layers,
         "attention_ms": attn_ms_mean,
         "append_ms": app_ms,
         "roofline": {
@@ -330,9 +345,10 @@ def run_ours(args, w, rank, world, local_rank):
             "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"],
             "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
             "peak_source": f"{peaks['source']} bf16 dense (burst)",
-            "kernel": "mla_attn_tc_kernel<192,32>",
-            "algorithmic_flops_per_launch": attn_fl,
-            "traffic": profiled_traffic("attn_tc_wan_traffic.json", "attn_tc.cu"),
+            "kernel": "mla_attn_tc_kernel<192,32,2>",
+            "algorithmic_flops_per_launch": attn_l,
+            "traffic": (profiled_traffic("attn_tc_wan_traffic.json", "attn_tc.cu")
+                        if w.batch == 1 else None),
         },
         "roofline_append": {
             "bound": "hbm", "kernel": "mla_append_tc_kernel<192,32>",
@@ -348,7 +364,7 @@ def run_ours(args, w, rank, world, local_rank):
             "ms_per_step": e2e_ms / e2e_steps, "steps": e2e_steps,
         },
         "clocks": clk.summary(),
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": 2 * w.layers * args.steps,
     }
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_oracle_sample(w, budget_s=args.cpu_budget)

@@ -44,6 +44,7 @@ class Workload:
     batch: int = 1
     last_frame: int = 21                  # frames_written after the timed chunk
     rms_eps: float = 1e-6
+    layers: int = 1                       # attention layers per benchmark step
 
     @property
     def tokens_per_frame(self):
@@ -69,6 +70,8 @@ WORKLOADS = {
     # Wan2.1-1.3B layer: 4680-token chunk against a full 21-frame window,
     # the paper's (6, 5, 5) RoPE pairs
     "wan": Workload("wan"),
+    # a full denoising step of the 30-block backbone: one Wan layer per block
+    "wan30": Workload("wan30", layers=30),
     # batch 4, positions advancing to latent frame 960 in a 21-frame ring
     "rollout": Workload("rollout", batch=4, last_frame=960),
 }
