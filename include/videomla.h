@@ -238,6 +238,22 @@ int mla_query_prologue_noalloc(const mla_config* cfg, const void* x, const void*
 int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* w_b, int Nq,
                           void* y, void* stream);
 
+/*
+ * Dense per-head attention: the baseline VideoMLA replaces, where every token
+ * caches K and V for every head, 2*n_h*d_h scalars (App. C.1; the dense rows
+ * of Table 1). Used for the d_c sweep's comparison (Table 5a); same window
+ * and query chunk as mla_attention_forward:
+ *     o_h = softmax_j(q_h . k_{h,j} / sqrt(head_dim)) v_{h,j}
+ *  q bf16 [batch][Nq][heads][head_dim] (RoPE already applied)
+ *  k, v bf16 [batch][heads][slots][head_dim] (k rotated); the first n_valid
+ *       slots of each head are read
+ *  o bf16 [batch][Nq][heads][head_dim]
+ * MLA_ERR_UNSUPPORTED unless head_dim is 64 or 128.
+ */
+int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void* k,
+                                const void* v, int slots, int n_valid, int Nq, void* o,
+                                void* stream);
+
 /* Human-readable name of a status code. */
 const char* mla_status_string(int status);
 

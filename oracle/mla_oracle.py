@@ -58,6 +58,7 @@ __all__ = [
     "softmax",
     "latent_attention",
     "reference_attention",
+    "dense_attention",
     "absorb_query",
     "absorb_output",
     "absorbed_query_matrices",
@@ -280,6 +281,19 @@ def reference_attention(x_q, pos_q, x_kv, pos_kv, w, head_dim, spec,
     if return_probs:
         out.append(p)
     return out[0] if len(out) == 1 else tuple(out)
+
+
+def dense_attention(q, k, v, head_dim):
+    """Dense per-head attention, the layout VideoMLA replaces (App. C.1).
+
+    q [Nq, H, d_h]; k, v [H, Nk, d_h] (RoPE already applied to q and k).
+    o_h = softmax(q_h k_h^T / sqrt(head_dim)) v_h.
+    """
+    q = np.asarray(q, dtype=np.float64)
+    k = np.asarray(k, dtype=np.float64)
+    v = np.asarray(v, dtype=np.float64)
+    s = np.einsum("nhd,hjd->nhj", q, k) / math.sqrt(head_dim)
+    return np.einsum("nhj,hjd->nhd", softmax(s, axis=-1), v)
 
 
 # --------------------------------------------------------------------------

@@ -389,6 +389,33 @@ int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* 
   return launch_output_projection(a);
 }
 
+int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void* k,
+                                const void* v, int slots, int n_valid, int Nq, void* o,
+                                void* stream) {
+  const int rc = check_config(cfg);
+  if (rc != MLA_OK) return rc;
+  if (!q || !k || !v || !o || Nq < 1 || slots < 1 || n_valid < 1 || n_valid > slots)
+    return MLA_ERR_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o)) return MLA_ERR_ARG;
+  DenseArgs a;
+  a.q = q;
+  a.k = k;
+  a.v = v;
+  a.o = o;
+  a.batch = cfg->batch;
+  a.nq = Nq;
+  a.heads = cfg->heads;
+  a.head_dim = cfg->head_dim;
+  a.slots = slots;
+  a.n_valid = n_valid;
+  a.scale_log2 =
+      static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(cfg->head_dim)));
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return launch_dense_attention_tc(a);
+}
+
 const char* mla_status_string(int status) {
   switch (status) {
     case MLA_OK: return "ok";

@@ -84,6 +84,18 @@ struct OutProjArgs {
   cudaStream_t stream;
 };
 
+// Dense per-head attention (the baseline cache layout).
+struct DenseArgs {
+  const void* q;        // bf16 [B][nq][H][head_dim]
+  const void* k;        // bf16 [B][H][slots][head_dim]
+  const void* v;        // bf16 [B][H][slots][head_dim]
+  void* o;              // bf16 [B][nq][H][head_dim]
+  int batch, nq, heads, head_dim, slots, n_valid;
+  float scale_log2;
+  int* status;
+  cudaStream_t stream;
+};
+
 // Each launcher returns MLA_OK, MLA_ERR_UNSUPPORTED or MLA_ERR_CUDA.
 int launch_attention_tc(const AttnArgs& a);
 int launch_attention_simt(const AttnArgs& a);
@@ -92,6 +104,7 @@ int launch_append_simt(const AppendArgs& a);
 int launch_absorb(const AbsorbArgs& a);
 int launch_query_prologue(const QueryArgs& a);
 int launch_output_projection(const OutProjArgs& a);
+int launch_dense_attention_tc(const DenseArgs& a);
 // Device address of the fixed no-allocation scratch on the current device.
 int query_scratch_address(void** out);
 

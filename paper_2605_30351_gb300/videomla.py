@@ -31,7 +31,7 @@ MLA_FLAG_SIMT = 2
 EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
-           "mla_query_prologue_noalloc", "mla_output_projection",
+           "mla_query_prologue_noalloc", "mla_output_projection", "mla_dense_attention_forward",
            "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
 
 
@@ -95,10 +95,12 @@ def load():
                                        VP, VP]
     lib.mla_output_projection.argtypes = [P(mla_config), VP, VP, I, VP, VP]
     lib.mla_query_prologue_noalloc.argtypes = [P(mla_config), VP, VP, VP, I, VP, VP, VP]
+    lib.mla_dense_attention_forward.argtypes = [P(mla_config), VP, VP, VP, I, I, I, VP, VP]
     for name in ("mla_rope_table_fill", "mla_config_check", "mla_cache_reset", "mla_cache_append",
                  "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
-                 "mla_query_prologue_noalloc", "mla_output_projection"):
+                 "mla_query_prologue_noalloc", "mla_output_projection",
+                 "mla_dense_attention_forward"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -291,6 +293,19 @@ def mla_output_projection(cfg, o_lat, w_b, y, stream=None):
                ctypes.byref(cfg), _dev(o_lat, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "o_lat"),
                _dev(w_b, bf, (cfg.hidden, cfg.heads * cfg.d_c), "w_b"), int(Nq),
                _dev(y, bf, (cfg.batch, Nq, cfg.hidden), "y"), _stream_ptr(stream)))
+
+
+def mla_dense_attention_forward(cfg, q, k, v, n_valid, o, stream=None):
+    """Dense per-head baseline: q [B, Nq, H, d_h], k/v [B, H, slots, d_h]."""
+    B, Nq, H, dh = cfg.batch, q.shape[1], cfg.heads, cfg.head_dim
+    slots = k.shape[2]
+    bf = torch.bfloat16
+    _check("mla_dense_attention_forward",
+           load().mla_dense_attention_forward(
+               ctypes.byref(cfg), _dev(q, bf, (B, Nq, H, dh), "q"),
+               _dev(k, bf, (B, H, slots, dh), "k"), _dev(v, bf, (B, H, slots, dh), "v"),
+               int(slots), int(n_valid), int(Nq), _dev(o, bf, (B, Nq, H, dh), "o"),
+               _stream_ptr(stream)))
 
 
 def mla_device_status(clear=True):

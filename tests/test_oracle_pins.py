@@ -399,3 +399,11 @@ def test_absorbed_matrices_apply_like_the_absorbed_maps():
     o_h = O.per_head_output_from_latent(o_lat, w_uv)
     np.testing.assert_allclose(y, o_h.reshape(4, -1) @ w_o.T, rtol=1e-12, atol=1e-12)
     np.testing.assert_allclose(O.absorb_output(o_lat, w_uv, w_o), y, rtol=1e-12, atol=1e-12)
+
+
+def test_dense_attention_is_sdpa():
+    """The dense baseline is torch's SDPA per head."""
+    rng = _rng(13)
+    q, k, v = rng.standard_normal((6, 3, 8)), rng.standard_normal((3, 10, 8)), rng.standard_normal((3, 10, 8))
+    ref = _sdpa(q.transpose(1, 0, 2), k, v).transpose(1, 0, 2)
+    np.testing.assert_allclose(O.dense_attention(q, k, v, 8), ref, rtol=1e-12, atol=1e-12)
