@@ -396,6 +396,231 @@ def run_reference(args, w, rank):
     }
 
 
+# ------------------------------------------------------- latent-size sweep
+def time_launches(fn, steps, warmup, stream):
+    """Median CUDA-event time (ms) of fn() over `steps` launches after `warmup`."""
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    ev[0].record(stream)
+    for i in range(steps):
+        fn()
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    return float(np.median([ev[i].elapsed_time(ev[i + 1]) for i in range(steps)]))
+
+
+def run_sweep(args, rank):
+    """Latent-size sweep (the d_c axis of Table 5, left; Sec. 3.3's cache sizes):
+    absorbed MLA attention for d_c in {64..512} x d_r in {32, 64} next to the
+    dense per-head baseline (12 x 128 K and V per token) at the same query
+    chunk and window; bytes per token, TFLOP/s and chunk latency. Shapes
+    without a tensor-core instance run the SIMT kernel and say so."""
+    from paper_2605_30351_gb300 import videomla as V
+
+    V.load()
+    stream = torch.cuda.current_stream()
+    base = synth.workload("wan")
+    peaks = load_peaks()
+    layers = 30
+    rows = []
+    for d_c in (64, 128, 192, 256, 512):
+        for d_r in (32, 64):
+            pairs = (6, 5, 5) if d_r == 32 else (12, 10, 10)
+            dims = (44, 42, 42) if d_r == 32 else (64, 64, 64)
+            w = base.with_(d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims)
+            cfg = V.make_config(w)
+            s = LayerSet(w, 7000 + d_c + d_r, V)
+            kind = "tcgen05"
+            try:
+                V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
+            except V.MlaError:
+                cfg.flags = V.MLA_FLAG_SIMT
+                s.cache.struct.cfg.flags = V.MLA_FLAG_SIMT
+                kind = "simt (no tensor-core instance for this shape)"
+            steps = args.steps if kind == "tcgen05" else 2
+            ms = time_launches(lambda: V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o,
+                                                               stream), steps, 2, stream)
+            fl = flops_per_layer(w)[0]
+            rows.append({
+                "layout": "mla", "d_c": d_c, "d_r": d_r, "kernel": kind,
+                "bytes_per_token_per_layer": 2 * (d_c + d_r),
+                "cache_gb_30_layers_21_frames": layers * w.slots * (d_c + d_r) * 2 / 1e9,
+                "compression_vs_dense": 2 * w.heads * w.head_dim / (d_c + d_r),
+                "ms_per_chunk_layer": ms, "tflops": fl / (ms * 1e-3) / 1e12,
+                "frac_of_measured_bf16_burst": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"],
+                "flop_per_row_key": 4 * d_c + 2 * d_r})
+            del s
+            torch.cuda.empty_cache()
+    # dense per-head baseline: q, k, v with d_h = 128, 12 heads, same window
+    w = base
+    cfg = V.make_config(w)
+    g = torch.Generator(device="cuda").manual_seed(11)
+    q = torch.randn(1, w.chunk_tokens, w.heads, w.head_dim, device="cuda", generator=g).to(torch.bfloat16)
+    k = torch.randn(1, w.heads, w.slots, w.head_dim, device="cuda", generator=g).to(torch.bfloat16)
+    v = torch.randn(1, w.heads, w.slots, w.head_dim, device="cuda", generator=g).to(torch.bfloat16)
+    o = torch.empty_like(q)
+    ms = time_launches(lambda: V.mla_dense_attention_forward(cfg, q, k, v, w.slots, o, stream),
+                       args.steps, 2, stream)
+    fl = 4.0 * w.chunk_tokens * w.heads * w.slots * w.head_dim
+    rows.append({
+        "layout": "dense", "d_h": w.head_dim, "kernel": "tcgen05",
+        "bytes_per_token_per_layer": 2 * 2 * w.heads * w.head_dim,
+        "cache_gb_30_layers_21_frames": layers * w.slots * 2 * w.heads * w.head_dim * 2 / 1e9,
+        "ms_per_chunk_layer": ms, "tflops": fl / (ms * 1e-3) / 1e12,
+        "frac_of_measured_bf16_burst": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"],
+        "flop_per_row_key": 4 * w.head_dim})
+    if rank != 0:
+        return None
+    return {"metric": "latent-size sweep: absorbed MLA attention vs dense per-head baseline",
+            "unit": "ms per chunk per layer", "data": "synthetic", "dtype": "bf16",
+            "config": {"workload": workload_desc(base) + "; d_c and d_r varied"},
+            "sweep": rows}
+
+
+# ------------------------------------------------------ memory-cap batch sweep
+B200_USABLE_GB = 180.0  # HBM of the B200 the paper's batch-scaling figure ran on
+
+
+def memcap_plan(w, layout, budget_bytes, layers=30):
+    """Largest batch whose attention-path state fits in `budget_bytes` (Sec. 4,
+    batch scaling under fixed memory: the caches decide when MHA runs out).
+
+    Per batch element: the caches of every layer for the whole window
+    (`layout` "mla": c and k_r, 2 (d_c + d_r) bytes per token per layer;
+    "dense": per-head K and V, 2 * 2 * H * d_h) plus one layer's chunk
+    activations in flight (x, positions, queries, attention output, y). Fixed:
+    every layer's projection weights. The rest of the DiT (FFN, norms) is not
+    counted."""
+    n, hid, H = w.chunk_tokens, w.hidden, w.heads
+    if layout == "mla":
+        cache_tok = 2 * (w.d_c + w.d_r)
+        q_row, o_row = H * (w.d_c + w.d_r) * 2, H * w.d_c * 2
+        weights = 2 * ((w.d_c + w.d_r) * hid + w.d_c + w.d_q * hid + w.d_q
+                       + H * (w.d_c + w.d_r) * w.d_q + hid * H * w.d_c)
+    else:
+        cache_tok = 2 * 2 * H * w.head_dim
+        q_row, o_row = H * w.head_dim * 2, H * w.head_dim * 2
+        weights = 2 * 4 * hid * H * w.head_dim
+    cache_b = layers * w.slots * cache_tok
+    act_b = n * (hid * 2 + 3 * 4 + q_row + o_row + hid * 2)
+    per_batch = cache_b + act_b
+    fixed = layers * weights
+    b_max = max(0, int((budget_bytes - fixed) // per_batch))
+    return {"cache_bytes_per_batch": cache_b, "activation_bytes_per_batch": act_b,
+            "weight_bytes": fixed, "per_batch_bytes": per_batch, "max_batch": b_max,
+            "bytes_at_max_batch": fixed + b_max * per_batch}
+
+
+def run_memcap(args, rank):
+    """Maximum batch of one chunk-against-window attention step under a fixed
+    HBM budget, dense per-head caches against latent caches at several d_c;
+    the plan is checked by allocating every layer's cache at that batch and
+    running one layer there (append and attention for the latent layout,
+    attention for the dense one)."""
+    from paper_2605_30351_gb300 import videomla as V
+
+    V.load()
+    stream = torch.cuda.current_stream()
+    base = synth.workload("wan")
+    layers = 30
+    budget = args.mem_budget_gb * 1e9
+    total = torch.cuda.mem_get_info()[1]
+    layouts = [("dense", base)] + [("mla", base.with_(d_c=dc)) for dc in (64, 128, 192, 256, 512)]
+    rows = []
+    g = torch.Generator(device="cuda").manual_seed(23)
+    for layout, w in layouts:
+        plan = memcap_plan(w, layout, budget, layers)
+        whole = memcap_plan(w, layout, total - 4e9, layers)
+        B = plan["max_batch"]
+        wb = w.with_(batch=B)
+        row = {"layout": layout, "d_c": w.d_c if layout == "mla" else None,
+               "d_r": w.d_r if layout == "mla" else None,
+               "gb_per_batch": plan["per_batch_bytes"] / 1e9,
+               "cache_gb_per_batch": plan["cache_bytes_per_batch"] / 1e9,
+               "max_batch": B, f"max_batch_{total / 1e9:.0f}gb_device": whole["max_batch"]}
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        before = torch.cuda.memory_allocated()
+        nq = w.chunk_tokens
+        if layout == "mla":
+            cfg = V.make_config(wb)
+            caches = [V.LatentCache(cfg) for _ in range(layers)]
+            x = torch.empty(B, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
+            pos = torch.empty(B, nq, 3, dtype=torch.int32, device="cuda")
+            q_c = torch.empty(B, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+            q_r = torch.empty(B, nq, w.heads, w.d_r, dtype=torch.bfloat16, device="cuda")
+            o = torch.empty(B, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+            y = torch.empty(B, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
+            wt = {k: v.cuda() for k, v in synth.draw_layer_weights(w, 29).items()}
+        else:
+            kv = [(torch.empty(B, w.heads, w.slots, w.head_dim, dtype=torch.bfloat16, device="cuda"),
+                   torch.empty(B, w.heads, w.slots, w.head_dim, dtype=torch.bfloat16, device="cuda"))
+                  for _ in range(layers)]
+            x = torch.empty(B, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
+            q = torch.empty(B, nq, w.heads, w.head_dim, dtype=torch.bfloat16, device="cuda")
+            o = torch.empty_like(q)
+            y = torch.empty_like(x)
+        used = torch.cuda.memory_allocated() - before
+        row["allocated_gb_at_max_batch"] = used / 1e9
+        row["fits_budget"] = bool(used <= budget)
+        fl_row = (4 * w.d_c + 2 * w.d_r) if layout == "mla" else 4 * w.head_dim
+        fl = 1.0 * B * nq * w.heads * w.slots * fl_row
+        tc = layout == "dense" or (w.d_c, w.d_r) in ((64, 32), (128, 32), (192, 32), (256, 32))
+        if B > 0 and tc:
+            if layout == "mla":
+                c0 = caches[0]
+                c0.c.normal_(generator=g)
+                c0.kr.normal_(generator=g)
+                c0.frames_written = w.window_frames
+                x.normal_(generator=g)
+                q_c.normal_(generator=g)
+                q_r.normal_(generator=g)
+                pos.copy_(synth.grid_positions(wb, w.window_frames - w.chunk_frames,
+                                               w.chunk_frames).to(pos.device))
+                first = w.window_frames - w.chunk_frames
+                t_app = time_launches(lambda: V.mla_cache_append(
+                    c0, x, wt["w_dkv"], wt["gamma_kv"], wt["w_kr"], pos, first, w.chunk_frames,
+                    stream), 3, 1, stream)
+                t_att = time_launches(lambda: V.mla_attention_forward(c0, q_c, q_r, pos, o, stream),
+                                      3, 1, stream)
+                row["append_ms_at_max_batch"] = t_app
+            else:
+                k0, v0 = kv[0]
+                k0.normal_(generator=g)
+                v0.normal_(generator=g)
+                q.normal_(generator=g)
+                cfg = V.make_config(wb)
+                t_att = time_launches(lambda: V.mla_dense_attention_forward(cfg, q, k0, v0, w.slots,
+                                                                            o, stream), 3, 1, stream)
+            row["attention_ms_at_max_batch"] = t_att
+            row["attention_tflops_at_max_batch"] = fl / (t_att * 1e-3) / 1e12
+            row["query_tokens_per_s_one_layer"] = B * nq / (t_att * 1e-3)
+            status = V.mla_device_status(clear=True)
+            if status != V.MLA_OK:
+                raise RuntimeError(f"device status {status} in the memory-cap run")
+        else:
+            row["attention_ms_at_max_batch"] = None
+            row["note"] = "allocation only: no tensor-core instance for this shape"
+        rows.append(row)
+        del x, o, y
+        if layout == "mla":
+            del caches, q_c, q_r, pos, wt
+        else:
+            del kv, q
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+    if rank != 0:
+        return None
+    return {"metric": "maximum batch under a fixed HBM budget: dense per-head vs latent caches",
+            "unit": "batch elements (one 4680-token chunk against a 21-frame window each)",
+            "data": "synthetic", "dtype": "bf16",
+            "config": {"workload": workload_desc(base) + f"; {layers} layers of caches; budget "
+                       f"{args.mem_budget_gb:g} GB (a B200's usable HBM) and the whole device"},
+            "memcap": rows}
+
+
 # -------------------------------------------------------------- distributed
 def barrier(world):
     if world > 1:
@@ -427,6 +652,10 @@ def main():
     ap.add_argument("--workload", default="wan")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", choices=["dc", "memcap"], default=None,
+                    help="dc: latent-size sweep next to the dense baseline; memcap: maximum "
+                         "batch under --mem-budget-gb (one JSON line each)")
+    ap.add_argument("--mem-budget-gb", type=float, default=B200_USABLE_GB)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -437,7 +666,11 @@ def main():
     if world > 1 and args.impl == "ours":
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
-    if args.impl == "reference":
+    if args.sweep == "dc":
+        out = run_sweep(args, rank)
+    elif args.sweep == "memcap":
+        out = run_memcap(args, rank)
+    elif args.impl == "reference":
         out = run_reference(args, w, rank)
     else:
         out = run_ours(args, w, rank, world, local_rank)
