@@ -40,6 +40,17 @@ notes of the repository):
       for every d_c.
   R5  Ring slot of token k of latent frame f: (f mod W_frames) * T + k
       (FIFO eviction, App. D.4).
+  R12 Long-rollout window (App. D.4): the first S latent frames (S = 1, the
+      sink) stay for good, the other W - S slots-frames hold the newest
+      W - S frames in FIFO order (W - S = 6), and the current chunk is among
+      them (it is appended before attention). Token k of frame f sits at
+      f * T + k for f < S, else (S + (f - S) mod (W - S)) * T + k; S = 0 is
+      the plain ring of R5.
+  R13 Window-relative RoPE (App. D.5): the cache keeps k^R unrotated; when a
+      window is assembled its held frames are numbered 0, 1, ... in temporal
+      order (sinks first) and that number is the temporal coordinate of their
+      keys and of the queries of those frames; (h, w) stay as given. Before
+      any eviction this is the absolute frame index.
 """
 
 import math
@@ -53,6 +64,10 @@ __all__ = [
     "rmsnorm",
     "ring_slot",
     "window_frames",
+    "sink_ring_slot",
+    "sink_window_frames",
+    "window_local_time",
+    "window_attention",
     "OracleCache",
     "cache_append",
     "softmax",
@@ -148,21 +163,56 @@ def window_frames(frames_written, window_frames):
     return list(range(first, frames_written))
 
 
-class OracleCache:
-    """Latent cache state: c [B, slots, d_c], k_rope [B, slots, d_r], frame ids."""
+# --------------------------------------------------------------------------
+# Sink + FIFO window and window-relative RoPE (App. D.4, D.5; R12, R13)
+# --------------------------------------------------------------------------
+def sink_ring_slot(frame, k, tokens_per_frame, window_frames, sink_frames):
+    """Slot of token k of latent frame `frame` when the first `sink_frames`
+    frames are kept for good and the later frames share the remaining
+    window_frames - sink_frames frame slots in FIFO order (reading R12)."""
+    if frame < sink_frames:
+        return frame * tokens_per_frame + k
+    local = window_frames - sink_frames
+    return (sink_frames + (frame - sink_frames) % local) * tokens_per_frame + k
 
-    def __init__(self, batch, tokens_per_frame, window_frames, d_c, d_r):
+
+def sink_window_frames(frames_written, window_frames, sink_frames):
+    """Frames held after `frames_written` in-order appends, in temporal order:
+    the sink frames, then the newest window_frames - sink_frames frames."""
+    sinks = list(range(min(sink_frames, frames_written)))
+    first_local = max(sink_frames, frames_written - (window_frames - sink_frames))
+    return sinks + list(range(first_local, frames_written))
+
+
+def window_local_time(frame, frames_written, window_frames, sink_frames):
+    """Temporal coordinate of a held frame inside the assembled window: its
+    index among the held frames in temporal order (reading R13). Raises
+    ValueError for a frame the window does not hold."""
+    return sink_window_frames(frames_written, window_frames, sink_frames).index(frame)
+
+
+class OracleCache:
+    """Latent cache state: c [B, slots, d_c], k [B, slots, d_r] (rotated at
+    append, or unrotated for the window path), the frame of every slot and
+    the (t, h, w) each slot's token was appended with."""
+
+    def __init__(self, batch, tokens_per_frame, window_frames, d_c, d_r, sink_frames=0):
         self.T = tokens_per_frame
         self.W = window_frames
+        self.S = sink_frames
         slots = tokens_per_frame * window_frames
         self.c = np.zeros((batch, slots, d_c))
         self.kr = np.zeros((batch, slots, d_r))
+        self.pos_of_slot = np.zeros((batch, slots, 3), dtype=np.int64)
         self.frame_of_slot = np.full(slots, -1, dtype=np.int64)
         self.frames_written = 0
 
+    def held_frames(self):
+        return sink_window_frames(self.frames_written, self.W, self.S)
+
     def valid_slots(self):
         """Slots that hold a frame of the current window (App. D.4)."""
-        held = set(window_frames(self.frames_written, self.W))
+        held = set(self.held_frames())
         return np.array([s for s in range(len(self.frame_of_slot))
                          if self.frame_of_slot[s] in held], dtype=np.int64)
 
@@ -176,7 +226,9 @@ def cache_append(cache, x, w_dkv, w_kr, pos, first_frame, n_frames,
     w_kr : [d_r, d]  decoupled RoPE key projection (Eq. krope)
     pos  : [B, n_frames*T, 3] (t, h, w) of each token
     Stores c = RMSNorm(W_dkv x) (reading R3) and k = RoPE3D(W_kr x, pos)
-    (reading R2) at the FIFO slots of frames first_frame .. first_frame+n_frames-1.
+    (reading R2), or k = W_kr x unrotated when spec is None (the paper's
+    storage, App. D.5), at the FIFO slots of frames
+    first_frame .. first_frame+n_frames-1 (readings R5, R12).
     """
     x = np.asarray(x, dtype=np.float64)
     B, n_tok, _ = x.shape
@@ -189,9 +241,10 @@ def cache_append(cache, x, w_dkv, w_kr, pos, first_frame, n_frames,
         k = rope3d(k, pos, spec)
     for n in range(n_tok):
         f = first_frame + n // cache.T
-        s = ring_slot(f, n % cache.T, cache.T, cache.W)
+        s = sink_ring_slot(f, n % cache.T, cache.T, cache.W, cache.S)
         cache.c[:, s, :] = c[:, n, :]
         cache.kr[:, s, :] = k[:, n, :]
+        cache.pos_of_slot[:, s, :] = np.asarray(pos)[:, n, :]
         cache.frame_of_slot[s] = f
     cache.frames_written = max(cache.frames_written, first_frame + n_frames)
     return c, k
@@ -236,6 +289,30 @@ def latent_attention(q_c, q_r, q_pos, keys_c, keys_k, head_dim, spec,
     p = softmax(s, axis=-1)
     o = np.einsum("nhj,jc->nhc", p, kc)
     return (o, p) if return_probs else o
+
+
+def window_attention(cache, b, q_c, q_r, q_pos, head_dim, spec):
+    """Attention of a query chunk over the assembled window of a cache that
+    stores k^R unrotated (App. D.4, D.5; readings R12, R13).
+
+    cache : OracleCache filled by cache_append(..., spec=None)
+    b     : batch element
+    q_c, q_r : [Nq, H, d_c], [Nq, H, d_r] as for latent_attention
+    q_pos : [Nq, 3] (t, h, w) with t the query token's absolute frame, which
+            the window must hold
+    Every held frame gets its window-local temporal coordinate; the cached
+    keys and the queries are rotated at those coordinates, then the scores
+    and outputs are those of latent_attention over the held slots.
+    """
+    slots = cache.valid_slots()
+    fw = cache.frames_written
+    key_pos = cache.pos_of_slot[b, slots].copy()
+    key_pos[:, 0] = [window_local_time(cache.frame_of_slot[s], fw, cache.W, cache.S)
+                     for s in slots]
+    k_rope = rope3d(cache.kr[b, slots], key_pos, spec)
+    q_local = np.array(q_pos, dtype=np.int64).copy()
+    q_local[:, 0] = [window_local_time(t, fw, cache.W, cache.S) for t in q_local[:, 0]]
+    return latent_attention(q_c, q_r, q_local, cache.c[b, slots], k_rope, head_dim, spec)
 
 
 def reference_attention(x_q, pos_q, x_kv, pos_kv, w, head_dim, spec,
