@@ -36,9 +36,12 @@ PROFILES = os.path.join(ROOT, "profiles")
 def workload_desc(w):
     layers = f"{w.layers} layers (distinct weights and caches), " if w.layers > 1 else ""
     pos = f"; latent frames up to {w.last_frame - 1} (ring wrapped)" if w.last_frame > w.window_frames else ""
+    frames = (f"{w.window_frames} frames: {w.sink_frames} sink + {w.window_frames - w.sink_frames}"
+              f" newest, k^R rotated at use at window-relative positions" if w.sink_frames
+              else f"{w.window_frames} frames")
     return (f"Wan2.1-1.3B attention layer: {w.chunk_tokens}-query chunk "
             f"({w.chunk_frames} latent frames of {w.grid_h}x{w.grid_w}) x {w.slots}-key window "
-            f"({w.window_frames} frames), {w.heads} heads, d_c={w.d_c}, d_r={w.d_r}, "
+            f"({frames}), {w.heads} heads, d_c={w.d_c}, d_r={w.d_r}, "
             f"batch {w.batch}; step = {layers}cache append + attention{pos}")
 
 
@@ -156,9 +159,23 @@ def cpu_oracle_sample(w, budget_s=12.0, seed=5, tokens_per_batch=8):
     wd, wk, g = f64(weights["w_dkv"]), f64(weights["w_kr"]), f64(weights["gamma_kv"])
     c, k = synth.draw_cache_rows(w, w.slots, seed + 1, batch=1)
     c, k = f64(c[0]), f64(k[0])
+    if w.sink_frames:
+        # the window oracle: a cache holding the sink frame and the newest
+        # frames with k^R unrotated, rotated at window-local times per call
+        win = O.OracleCache(1, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r,
+                            sink_frames=w.sink_frames)
+        T = w.tokens_per_frame
+        first_local = w.last_frame - (w.window_frames - w.sink_frames)
+        for f in list(range(w.sink_frames)) + list(range(first_local, w.last_frame)):
+            s0 = O.sink_ring_slot(f, 0, T, w.window_frames, w.sink_frames)
+            win.frame_of_slot[s0:s0 + T] = f
+            win.pos_of_slot[0, s0:s0 + T] = synth.grid_positions(w, f, 1, batch=1)[0].numpy()
+        win.c[0], win.kr[0] = c, k
+        win.frames_written = w.last_frame
     q_c, q_r = synth.draw_queries(w, w.chunk_tokens, seed + 2, batch=1)
     x = synth.draw_tokens(w, w.chunk_tokens, seed + 3, batch=1)
-    pos = synth.grid_positions(w, w.window_frames - w.chunk_frames, w.chunk_frames, batch=1)
+    pos = synth.grid_positions(w, (w.last_frame if w.sink_frames else w.window_frames)
+                               - w.chunk_frames, w.chunk_frames, batch=1)
     q_c, q_r, x, pos = f64(q_c[0]), f64(q_r[0]), f64(x), pos.numpy()
     step = tokens_per_batch
     done = 0
@@ -170,8 +187,12 @@ def cpu_oracle_sample(w, budget_s=12.0, seed=5, tokens_per_batch=8):
         n = sl.stop - sl.start
         oc = O.OracleCache(1, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r)
         oc.T = n  # one partial "frame" of n tokens: the same arithmetic per token
-        O.cache_append(oc, x[:, sl], wd, wk, pos[:, sl], 0, 1, gamma=g, eps=w.rms_eps, spec=spec)
-        O.latent_attention(q_c[sl], q_r[sl], pos[0, sl], c, k, w.head_dim, spec)
+        O.cache_append(oc, x[:, sl], wd, wk, pos[:, sl], 0, 1, gamma=g, eps=w.rms_eps,
+                       spec=None if w.sink_frames else spec)
+        if w.sink_frames:
+            O.window_attention(win, 0, q_c[sl], q_r[sl], pos[0, sl], w.head_dim, spec)
+        else:
+            O.latent_attention(q_c[sl], q_r[sl], pos[0, sl], c, k, w.head_dim, spec)
         fl += 2.0 * n * w.hidden * (w.d_c + w.d_r)
         fl += O.latent_attention_flops(n * w.heads, w.slots, w.d_c, w.d_r)
         done += n
@@ -213,6 +234,12 @@ class LayerSet:
         self.q_c, self.q_r = q_c.cuda(), q_r.cuda()
         self.o = torch.empty(w.batch, w.chunk_tokens, w.heads, w.d_c, dtype=torch.bfloat16,
                              device="cuda")
+        # long-rollout window (sink frames, k^R unrotated): assembled per call
+        self.window = w.sink_frames > 0
+        if self.window:
+            self.hw = synth.frame_coords(w).cuda()
+            self.ws = torch.empty(V.mla_window_workspace_bytes(self.cache.cfg, w.chunk_tokens),
+                                  dtype=torch.uint8, device="cuda")
 
 
 def run_ours(args, w, rank, world, local_rank):
@@ -230,11 +257,14 @@ def run_ours(args, w, rank, world, local_rank):
     def layer(s, ev=None):
         if ev is not None:
             ev[0].record(stream)
-        V.mla_cache_append(s.cache, s.x, s.w_dkv, s.gamma, s.w_kr, s.pos, s.first,
-                           w.chunk_frames, stream)
+        V.mla_cache_append(s.cache, s.x, s.w_dkv, s.gamma, s.w_kr, None if s.window else s.pos,
+                           s.first, w.chunk_frames, stream)
         if ev is not None:
             ev[1].record(stream)
-        V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
+        if s.window:
+            V.mla_attention_window_forward(s.cache, s.q_c, s.q_r, s.pos, s.hw, s.ws, s.o, stream)
+        else:
+            V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
         if ev is not None:
             ev[2].record(stream)
 
@@ -345,7 +375,8 @@ def run_ours(args, w, rank, world, local_rank):
             "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"],
             "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
             "peak_source": f"{peaks['source']} bf16 dense (burst)",
-            "kernel": "mla_attn_tc_kernel<192,32,2>",
+            "kernel": ("window_assemble_kernel + mla_attn_tc_kernel<192,32,2> (events around both)"
+                       if w.sink_frames else "mla_attn_tc_kernel<192,32,2>"),
             "algorithmic_flops_per_launch": attn_l,
             "traffic": (profiled_traffic("attn_tc_wan_traffic.json", "attn_tc.cu")
                         if w.batch == 1 else None),
@@ -364,7 +395,7 @@ def run_ours(args, w, rank, world, local_rank):
             "ms_per_step": e2e_ms / e2e_steps, "steps": e2e_steps,
         },
         "clocks": clk.summary(),
-        "gpu_launches": 2 * w.layers * args.steps,
+        "gpu_launches": (3 if w.sink_frames else 2) * w.layers * args.steps,
     }
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_oracle_sample(w, budget_s=args.cpu_budget)

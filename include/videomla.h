@@ -39,6 +39,8 @@ extern "C" {
 /* cfg.flags */
 #define MLA_FLAG_NO_RMSNORM 1u   /* store c^KV = W_dkv x without RMSNorm (App. D.2 off) */
 #define MLA_FLAG_SIMT 2u         /* use the plain SIMT debug kernels (no tensor cores) */
+#define MLA_FLAG_ROTATE_AT_USE 4u /* cache k^R unrotated; attend with
+                                     mla_attention_window_forward (App. D.5) */
 
 /*
  * Shape of one VideoMLA attention layer (Sec. 3; App. D.2-D.4).
@@ -57,10 +59,14 @@ extern "C" {
  *  rope_theta      RoPE base (10000)
  *  rope_table_len  positions per axis the table covers (1024, App. C.1)
  *  tokens_per_frame T, tokens of one latent frame (30*52 = 1560, App. D.1)
- *  window_frames   W, latent frames the ring holds (21, Sec. 1 / App. D.4)
+ *  window_frames   W, latent frames the cache holds (21, Sec. 1 / App. D.4;
+ *                  7 = 1 sink + 6 local for long rollouts, App. D.4)
  *  batch           B, independent sequences, each with its own ring
  *  rms_eps         RMSNorm epsilon (1e-6)
  *  flags           MLA_FLAG_*
+ *  sink_frames     S, leading latent frames that are never evicted (0 for the
+ *                  plain 21-frame ring, 1 for the long-rollout window of
+ *                  App. D.4); 0 <= S < W
  */
 typedef struct mla_config {
   int hidden;
@@ -78,20 +84,23 @@ typedef struct mla_config {
   int batch;
   float rms_eps;
   unsigned flags;
+  int sink_frames;
 } mla_config;
 
 /*
  * The sliding-window latent cache (App. D.4). Caller-owned device buffers:
  *  c          bf16 [batch][window_frames*tokens_per_frame][d_c]   latent c^KV
- *  kr         bf16 [batch][window_frames*tokens_per_frame][d_r]   rotated k^R
+ *  kr         bf16 [batch][window_frames*tokens_per_frame][d_r]   k^R, rotated
+ *             at append, or unrotated with MLA_FLAG_ROTATE_AT_USE
  *  rope_table fp32 [rope_table_len][d_r/2][2] = (cos, sin) of position p
  *             times the pair's frequency; fill it with mla_rope_table_fill()
  *             and copy it to the device.
  *  frames_written  number of latent frames appended so far (advanced by
  *             mla_cache_append on the host; reset by mla_cache_reset).
- * Token k of latent frame f lives in slot (f mod window_frames)*T + k
- * (FIFO eviction, App. D.4). Slots of frames that were never written are
- * not read.
+ * Token k of latent frame f lives in slot f*T + k if f < S (a sink frame),
+ * else in slot (S + (f - S) mod (W - S))*T + k: the frames after the sinks
+ * share W - S frame slots in FIFO order (App. D.4). With S = 0 this is the
+ * ring (f mod W)*T + k. Slots of frames that were never written are not read.
  */
 typedef struct mla_cache {
   void* c;
@@ -131,10 +140,13 @@ int mla_cache_reset(mla_cache* cache, void* stream);
  *  gamma_kv bf16 [d_c] RMSNorm weight, or NULL for ones
  *  w_kr     bf16 [d_r][hidden]        decoupled RoPE key projection
  *  pos      int32 [batch][n_frames*T][3]  (t, h, w) of every token; each
- *           coordinate must lie in [0, rope_table_len) (device-checked)
+ *           coordinate must lie in [0, rope_table_len) (device-checked).
+ *           Not read (may be NULL) with MLA_FLAG_ROTATE_AT_USE.
  * The positional key is rotated here with the absolute positions given;
- * the scores only depend on position differences, so this matches
- * rotating at use with window-relative coordinates (Sec. 3.2, App. D.5).
+ * for a contiguous window the scores only depend on position differences,
+ * so this matches rotating at use with window-relative coordinates
+ * (Sec. 3.2, App. D.5). With MLA_FLAG_ROTATE_AT_USE the cache keeps
+ * k = W_kr x unrotated, the paper's own storage (App. D.5).
  * Rules: 1 <= n_frames <= window_frames (else MLA_ERR_RANGE);
  * 0 <= first_frame <= frames_written <= first_frame + n_frames (no gap, and
  * the range reaches the newest frame: extend the window or rewrite the
@@ -158,11 +170,44 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv,
  * Valid slots: the first min(frames_written, W)*T slots before the ring
  * first wraps, all slots after. The query chunk is taken to be the newest
  * chunk, so the chunk-causal mask (App. D.4) keeps every valid slot.
- * MLA_ERR_ARG if no slot is valid or Nq < 1.
+ * MLA_ERR_ARG if no slot is valid, Nq < 1, or the cache keeps k^R unrotated
+ * (MLA_FLAG_ROTATE_AT_USE: use mla_attention_window_forward).
  */
 int mla_attention_forward(const mla_cache* cache, const void* q_c,
                           const void* q_r, const int* q_pos, int Nq,
                           void* o_lat, void* stream);
+
+/* Bytes of caller-owned device workspace mla_attention_window_forward needs
+ * for Nq query tokens per batch element (0 on a bad config). */
+unsigned long long mla_window_workspace_bytes(const mla_config* cfg, int Nq);
+
+/*
+ * Attention over the assembled window of a cache that keeps k^R unrotated
+ * (MLA_FLAG_ROTATE_AT_USE), with window-relative RoPE (App. D.4, D.5):
+ *  1. the held frames (the S sinks, then the newest frames in temporal
+ *     order) are numbered 0, 1, ...; that number is the temporal coordinate
+ *     of every key of the frame, which is rotated by RoPE3D at
+ *     (local t, h, w) into the workspace;
+ *  2. each query's absolute frame q_pos[.][0] is mapped to the local number
+ *     of that frame (the frame must be held: the current chunk is appended
+ *     first), (h, w) unchanged;
+ *  3. the same absorbed-form attention as mla_attention_forward runs over
+ *     the valid slots with the rotated window keys.
+ * Before any eviction local and absolute times agree. Arguments as for
+ * mla_attention_forward, plus:
+ *  frame_hw  int32 [tokens_per_frame][2]: (h, w) of token k of every latent
+ *            frame (the latent grid is the same for all frames); each must
+ *            lie in [0, rope_table_len) (device-checked)
+ *  workspace device memory of at least mla_window_workspace_bytes(cfg, Nq)
+ *            bytes, 16-byte aligned, owned by the caller (scratch)
+ * A query frame the window does not hold is recorded as MLA_ERR_RANGE in
+ * the device status (its rows use local time 0). MLA_ERR_ARG unless the
+ * cache has MLA_FLAG_ROTATE_AT_USE.
+ */
+int mla_attention_window_forward(const mla_cache* cache, const void* q_c, const void* q_r,
+                                 const int* q_pos, int Nq, const int* frame_hw,
+                                 void* workspace, unsigned long long workspace_bytes,
+                                 void* o_lat, void* stream);
 
 /*
  * Load-time weight absorption (App. E, Eqs. absorb-q and absorb-v), computed

@@ -74,7 +74,62 @@ int check_config(const mla_config* c) {
   if (c->d_c % 8 != 0 || c->d_r % 8 != 0 || c->hidden % 8 != 0) return MLA_ERR_ARG;
   const long long slots = static_cast<long long>(c->tokens_per_frame) * c->window_frames;
   if (slots > (1ll << 30)) return MLA_ERR_ARG;
+  if (c->sink_frames < 0 || c->sink_frames >= c->window_frames) return MLA_ERR_ARG;
   return MLA_OK;
+}
+
+int fail_cuda(cudaError_t e);
+
+// Valid slots: the first min(frames_written, W) frame slots (contiguous from
+// 0 before the first eviction, all slots after).
+long long valid_slots(const mla_cache& cache) {
+  const mla_config& c = cache.cfg;
+  const long long held = cache.frames_written < c.window_frames ? cache.frames_written
+                                                                 : c.window_frames;
+  return held * c.tokens_per_frame;
+}
+
+bool rotate_at_use(const mla_config& c) { return (c.flags & MLA_FLAG_ROTATE_AT_USE) != 0; }
+
+// Absorbed-form attention over the valid slots, with the given positional
+// keys and query positions.
+int run_attention(const mla_cache* cache, const void* q_c, const void* q_r, const int* q_pos,
+                  int Nq, const void* kr, void* o_lat, cudaStream_t stream) {
+  const mla_config& c = cache->cfg;
+  const long long n_valid = valid_slots(*cache);
+  if (n_valid < 1) return MLA_ERR_ARG;
+  const long long rows = static_cast<long long>(Nq) * c.heads;
+  if (rows > (1ll << 30)) return MLA_ERR_ARG;
+  AttnArgs a;
+  a.q_c = q_c;
+  a.q_r = q_r;
+  a.q_pos = q_pos;
+  a.rope = static_cast<const float*>(cache->rope_table);
+  a.c = cache->c;
+  a.kr = kr;
+  a.o = o_lat;
+  a.batch = c.batch;
+  a.rows = static_cast<int>(rows);
+  a.heads = c.heads;
+  a.slots = c.tokens_per_frame * c.window_frames;
+  a.n_valid = static_cast<int>(n_valid);
+  a.d_c = c.d_c;
+  a.d_r = c.d_r;
+  a.rope_len = c.rope_table_len;
+  a.pairs_t = c.rope_pairs_t;
+  a.pairs_h = c.rope_pairs_h;
+  a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c.head_dim)));
+  a.status = device_status_ptr();
+  a.stream = stream;
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return (c.flags & MLA_FLAG_SIMT) ? launch_attention_simt(a) : launch_attention_tc(a);
+}
+
+unsigned long long round256(unsigned long long v) { return (v + 255) / 256 * 256; }
+
+unsigned long long window_kr_bytes(const mla_config& c) {
+  return round256(static_cast<unsigned long long>(c.batch) * c.tokens_per_frame *
+                  c.window_frames * c.d_r * 2);
 }
 
 int fail_cuda(cudaError_t e) {
@@ -174,7 +229,8 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv, const v
   int rc = check_config(&cache->cfg);
   if (rc != MLA_OK) return rc;
   const mla_config& c = cache->cfg;
-  if (!cache->c || !cache->kr || !cache->rope_table || !x || !w_dkv || !w_kr || !pos)
+  const bool rotate = !rotate_at_use(c);
+  if (!cache->c || !cache->kr || !cache->rope_table || !x || !w_dkv || !w_kr || (rotate && !pos))
     return MLA_ERR_ARG;
   if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(x) || !aligned16(w_dkv) ||
       !aligned16(w_kr) || !aligned16(cache->rope_table) || (gamma_kv && !aligned16(gamma_kv)) ||
@@ -189,7 +245,7 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv, const v
   a.w_dkv = w_dkv;
   a.gamma = gamma_kv;
   a.w_kr = w_kr;
-  a.pos = pos;
+  a.pos = rotate ? pos : nullptr;
   a.rope = static_cast<const float*>(cache->rope_table);
   a.c = cache->c;
   a.kr = cache->kr;
@@ -201,6 +257,8 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv, const v
   a.slots = c.tokens_per_frame * c.window_frames;
   a.tokens_per_frame = c.tokens_per_frame;
   a.window_frames = c.window_frames;
+  a.sink_frames = c.sink_frames;
+  a.rotate = rotate ? 1 : 0;
   a.first_frame = first_frame;
   a.rope_len = c.rope_table_len;
   a.pairs_t = c.rope_pairs_t;
@@ -228,36 +286,60 @@ int mla_attention_forward(const mla_cache* cache, const void* q_c, const void* q
       !aligned16(o_lat) || !aligned16(cache->rope_table) ||
       (reinterpret_cast<uintptr_t>(q_pos) & 3u))
     return MLA_ERR_ARG;
-  if (Nq < 1) return MLA_ERR_ARG;
-  const long long held = cache->frames_written < c.window_frames ? cache->frames_written
-                                                                  : c.window_frames;
-  const long long n_valid = held * c.tokens_per_frame;
+  if (Nq < 1 || rotate_at_use(c)) return MLA_ERR_ARG;
+  return run_attention(cache, q_c, q_r, q_pos, Nq, cache->kr, o_lat,
+                       static_cast<cudaStream_t>(stream));
+}
+
+unsigned long long mla_window_workspace_bytes(const mla_config* cfg, int Nq) {
+  if (check_config(cfg) != MLA_OK || Nq < 1) return 0;
+  return window_kr_bytes(*cfg) + static_cast<unsigned long long>(cfg->batch) * Nq * 3 * 4;
+}
+
+int mla_attention_window_forward(const mla_cache* cache, const void* q_c, const void* q_r,
+                                 const int* q_pos, int Nq, const int* frame_hw, void* workspace,
+                                 unsigned long long workspace_bytes, void* o_lat, void* stream) {
+  if (!cache) return MLA_ERR_ARG;
+  int rc = check_config(&cache->cfg);
+  if (rc != MLA_OK) return rc;
+  const mla_config& c = cache->cfg;
+  if (!rotate_at_use(c) || Nq < 1) return MLA_ERR_ARG;
+  if (!cache->c || !cache->kr || !cache->rope_table || !q_c || !q_r || !q_pos || !o_lat ||
+      !frame_hw || !workspace)
+    return MLA_ERR_ARG;
+  if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(q_c) || !aligned16(q_r) ||
+      !aligned16(o_lat) || !aligned16(cache->rope_table) || !aligned16(workspace) ||
+      (reinterpret_cast<uintptr_t>(q_pos) & 3u) || (reinterpret_cast<uintptr_t>(frame_hw) & 3u))
+    return MLA_ERR_ARG;
+  if (workspace_bytes < mla_window_workspace_bytes(&c, Nq)) return MLA_ERR_ARG;
+  const long long n_valid = valid_slots(*cache);
   if (n_valid < 1) return MLA_ERR_ARG;
-  const long long rows = static_cast<long long>(Nq) * c.heads;
-  if (rows > (1ll << 30)) return MLA_ERR_ARG;
-  AttnArgs a;
-  a.q_c = q_c;
-  a.q_r = q_r;
-  a.q_pos = q_pos;
-  a.rope = static_cast<const float*>(cache->rope_table);
-  a.c = cache->c;
-  a.kr = cache->kr;
-  a.o = o_lat;
-  a.batch = c.batch;
-  a.rows = static_cast<int>(rows);
-  a.heads = c.heads;
-  a.slots = c.tokens_per_frame * c.window_frames;
-  a.n_valid = static_cast<int>(n_valid);
-  a.d_c = c.d_c;
-  a.d_r = c.d_r;
-  a.rope_len = c.rope_table_len;
-  a.pairs_t = c.rope_pairs_t;
-  a.pairs_h = c.rope_pairs_h;
-  a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c.head_dim)));
-  a.status = device_status_ptr();
-  a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
-  return (c.flags & MLA_FLAG_SIMT) ? launch_attention_simt(a) : launch_attention_tc(a);
+  WindowArgs w;
+  w.kr = cache->kr;
+  w.q_pos = q_pos;
+  w.frame_hw = frame_hw;
+  w.rope = static_cast<const float*>(cache->rope_table);
+  w.kr_rot = workspace;
+  w.q_pos_local = reinterpret_cast<int*>(static_cast<unsigned char*>(workspace) +
+                                         window_kr_bytes(c));
+  w.batch = c.batch;
+  w.nq = Nq;
+  w.slots = c.tokens_per_frame * c.window_frames;
+  w.n_valid = static_cast<int>(n_valid);
+  w.T = c.tokens_per_frame;
+  w.W = c.window_frames;
+  w.S = c.sink_frames;
+  w.d_r = c.d_r;
+  w.frames_written = cache->frames_written;
+  w.rope_len = c.rope_table_len;
+  w.pairs_t = c.rope_pairs_t;
+  w.pairs_h = c.rope_pairs_h;
+  w.status = device_status_ptr();
+  w.stream = static_cast<cudaStream_t>(stream);
+  if (!w.status) return fail_cuda(cudaGetLastError());
+  rc = launch_window_assemble(w);
+  if (rc != MLA_OK) return rc;
+  return run_attention(cache, q_c, q_r, w.q_pos_local, Nq, w.kr_rot, o_lat, w.stream);
 }
 
 int mla_absorb_weights(const mla_config* cfg, const void* w_uq, const void* w_uk, const void* w_qr,

@@ -8,8 +8,10 @@
 //              [128 x (d_c + d_r)] fp32 accumulator (a single N = 224 MMA per
 //              K step at the paper's shape).
 //   warps 2-5  epilogue, thread i = token i: RMSNorm over the d_c columns in
-//              fp32, gamma, RoPE3D on the d_r columns, bf16, 16-byte stores
-//              into the token's ring slot (f mod W) * T + k.
+//              fp32, gamma, RoPE3D on the d_r columns (skipped when the
+//              cache keeps k^R unrotated), bf16, 16-byte stores into the
+//              token's slot: (f mod W) * T + k, or with S sink frames f * T + k
+//              for f < S and (S + (f - S) mod (W - S)) * T + k after them.
 #include <cmath>
 
 #include "internal.h"
@@ -49,9 +51,9 @@ struct AppendKParams {
   const float2* rope;
   __nv_bfloat16* c;
   __nv_bfloat16* kr;
-  int n_tok, k_blocks, slots, T, W;
+  int n_tok, k_blocks, slots, T, W, S;
   long long first_frame;
-  int rope_len, pairs_t, pairs_h, use_rmsnorm;
+  int rope_len, pairs_t, pairs_h, use_rmsnorm, rotate;
   float eps;
   int* status;
 };
@@ -179,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
       const long long f = p.first_frame + n / p.T;
-      slot_of[r] = row_ok ? (f % p.W) * p.T + n % p.T : -1;
+      slot_of[r] = row_ok ? frame_base_slot(f, p.T, p.W, p.S) + n % p.T : -1;
       uint8_t* srow = stage_out + r * S::kOutStride;
       // pass 2: gamma * c / rms -> bf16
 #pragma unroll 1
@@ -204,9 +206,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           *reinterpret_cast<uint4*>(srow + cb * 64 + i * 16) =
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
-      // positional key: RoPE3D at the token's (t, h, w)
+      // positional key: RoPE3D at the token's (t, h, w), or unrotated
       int pa[3] = {0, 0, 0};
-      if (row_ok) {
+      if (row_ok && p.rotate) {
         const int* pp = p.pos + (static_cast<size_t>(b) * p.n_tok + n) * 3;
         pa[0] = __ldg(pp);
         pa[1] = __ldg(pp + 1);
@@ -230,7 +232,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int ps = pr < p.pairs_t ? pa[0] : (pr < p.pairs_t + p.pairs_h ? pa[1] : pa[2]);
           const float2 cs = __ldg(p.rope + static_cast<size_t>(ps) * (DR / 2) + pr);
           const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
-          pk[i] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
+          pk[i] = p.rotate ? pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x)
+                           : pack_bf16x2(x0, x1);
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i)
@@ -293,6 +296,8 @@ int launch_tc(const AppendArgs& a) {
   kp.slots = a.slots;
   kp.T = a.tokens_per_frame;
   kp.W = a.window_frames;
+  kp.S = a.sink_frames;
+  kp.rotate = a.rotate;
   kp.first_frame = a.first_frame;
   kp.rope_len = a.rope_len;
   kp.pairs_t = a.pairs_t;

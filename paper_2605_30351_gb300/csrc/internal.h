@@ -8,6 +8,13 @@
 
 namespace vmla {
 
+// First slot of latent frame f: sink frames (f < S) keep slot f*T for good,
+// later frames share the W - S remaining frame slots in FIFO order
+// (App. D.4). With S = 0 this is the ring (f mod W)*T.
+__host__ __device__ inline long long frame_base_slot(long long f, int T, int W, int S) {
+  return (f < S ? f : S + (f - S) % (W - S)) * static_cast<long long>(T);
+}
+
 // One attention launch: every (token, head) row of the chunk against the
 // valid slots of its batch element's window.
 struct AttnArgs {
@@ -36,10 +43,11 @@ struct AppendArgs {
   void* c;              // bf16 [B][slots][d_c]
   void* kr;             // bf16 [B][slots][d_r]
   int batch, n_tok, hidden, d_c, d_r, slots;
-  int tokens_per_frame, window_frames;
+  int tokens_per_frame, window_frames, sink_frames;
   long long first_frame;
   int rope_len, pairs_t, pairs_h;
   int use_rmsnorm;
+  int rotate;           // 0: store W_kr x unrotated (pos is not read)
   float eps;
   int* status;
   cudaStream_t stream;
@@ -96,6 +104,22 @@ struct DenseArgs {
   cudaStream_t stream;
 };
 
+// Window assembly for rotate-at-use caches (App. D.5): rotated keys of the
+// valid slots at window-local times, and local query positions.
+struct WindowArgs {
+  const void* kr;       // bf16 [B][slots][d_r] unrotated k^R
+  const int* q_pos;     // int32 [B][nq][3] absolute (t, h, w)
+  const int* frame_hw;  // int32 [T][2]
+  const float* rope;    // fp32 [L][d_r/2][2]
+  void* kr_rot;         // out bf16 [B][slots][d_r] (first n_valid slots written)
+  int* q_pos_local;     // out int32 [B][nq][3]
+  int batch, nq, slots, n_valid, T, W, S, d_r;
+  long long frames_written;
+  int rope_len, pairs_t, pairs_h;
+  int* status;
+  cudaStream_t stream;
+};
+
 // Each launcher returns MLA_OK, MLA_ERR_UNSUPPORTED or MLA_ERR_CUDA.
 int launch_attention_tc(const AttnArgs& a);
 int launch_attention_simt(const AttnArgs& a);
@@ -105,6 +129,7 @@ int launch_absorb(const AbsorbArgs& a);
 int launch_query_prologue(const QueryArgs& a);
 int launch_output_projection(const OutProjArgs& a);
 int launch_dense_attention_tc(const DenseArgs& a);
+int launch_window_assemble(const WindowArgs& a);
 // Device address of the fixed no-allocation scratch on the current device.
 int query_scratch_address(void** out);
 

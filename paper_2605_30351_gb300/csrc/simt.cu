@@ -21,9 +21,9 @@ __global__ void append_simt_kernel(const __nv_bfloat16* __restrict__ x,
                                    const __nv_bfloat16* __restrict__ w_kr,
                                    const int* __restrict__ pos, const float2* __restrict__ rope,
                                    __nv_bfloat16* c, __nv_bfloat16* kr, int n_tok, int hidden,
-                                   int d_c, int d_r, int slots, int T, int W,
+                                   int d_c, int d_r, int slots, int T, int W, int S,
                                    long long first_frame, int rope_len, int pairs_t, int pairs_h,
-                                   int use_rmsnorm, float eps, int* status) {
+                                   int use_rmsnorm, int rotate, float eps, int* status) {
   extern __shared__ float sh[];  // hidden floats of x, then d_c + d_r outputs
   float* xs = sh;
   float* ys = sh + hidden;
@@ -55,11 +55,17 @@ __global__ void append_simt_kernel(const __nv_bfloat16* __restrict__ x,
   __syncthreads();
   const float inv = use_rmsnorm ? rsqrtf(red[0] / d_c + eps) : 1.f;
   const long long f = first_frame + n / T;
-  const long long slot = (f % W) * T + n % T;
+  const long long slot = frame_base_slot(f, T, W, S) + n % T;
   __nv_bfloat16* cd = c + (static_cast<size_t>(b) * slots + slot) * d_c;
   for (int col = threadIdx.x; col < d_c; col += blockDim.x) {
     const float g = gamma ? __bfloat162float(gamma[col]) : 1.f;
     cd[col] = __float2bfloat16_rn(ys[col] * inv * g);
+  }
+  __nv_bfloat16* kd = kr + (static_cast<size_t>(b) * slots + slot) * d_r;
+  if (!rotate) {  // the paper's storage: k^R = W_kr x, rotated when the window is assembled
+    for (int col = threadIdx.x; col < d_r; col += blockDim.x)
+      kd[col] = __float2bfloat16_rn(ys[d_c + col]);
+    return;
   }
   const int* pp = pos + (static_cast<size_t>(b) * n_tok + n) * 3;
   int pa[3] = {pp[0], pp[1], pp[2]};
@@ -68,7 +74,6 @@ __global__ void append_simt_kernel(const __nv_bfloat16* __restrict__ x,
       if (threadIdx.x == 0) record_status(status, MLA_ERR_RANGE);
       pa[a] = 0;
     }
-  __nv_bfloat16* kd = kr + (static_cast<size_t>(b) * slots + slot) * d_r;
   for (int pr = threadIdx.x; pr < d_r / 2; pr += blockDim.x) {
     const int ps = pr < pairs_t ? pa[0] : (pr < pairs_t + pairs_h ? pa[1] : pa[2]);
     const float2 cs = rope[static_cast<size_t>(ps) * (d_r / 2) + pr];
@@ -159,8 +164,8 @@ int launch_append_simt(const AppendArgs& a) {
       static_cast<const __nv_bfloat16*>(a.gamma), static_cast<const __nv_bfloat16*>(a.w_kr),
       a.pos, reinterpret_cast<const float2*>(a.rope), static_cast<__nv_bfloat16*>(a.c),
       static_cast<__nv_bfloat16*>(a.kr), a.n_tok, a.hidden, a.d_c, a.d_r, a.slots,
-      a.tokens_per_frame, a.window_frames, a.first_frame, a.rope_len, a.pairs_t, a.pairs_h,
-      a.use_rmsnorm, a.eps, a.status);
+      a.tokens_per_frame, a.window_frames, a.sink_frames, a.first_frame, a.rope_len, a.pairs_t,
+      a.pairs_h, a.use_rmsnorm, a.rotate, a.eps, a.status);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);

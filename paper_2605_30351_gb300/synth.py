@@ -21,7 +21,7 @@ import numpy as np
 import torch
 
 __all__ = ["Workload", "WORKLOADS", "workload", "bf16", "draw_layer_weights",
-           "draw_tokens", "grid_positions", "draw_queries", "draw_cache_rows"]
+           "draw_tokens", "grid_positions", "frame_coords", "draw_queries", "draw_cache_rows"]
 
 
 @dataclass(frozen=True)
@@ -45,6 +45,7 @@ class Workload:
     last_frame: int = 21                  # frames_written after the timed chunk
     rms_eps: float = 1e-6
     layers: int = 1                       # attention layers per benchmark step
+    sink_frames: int = 0                  # frames never evicted (long-rollout window)
 
     @property
     def tokens_per_frame(self):
@@ -74,6 +75,9 @@ WORKLOADS = {
     "wan30": Workload("wan30", layers=30),
     # batch 4, positions advancing to latent frame 960 in a 21-frame ring
     "rollout": Workload("rollout", batch=4, last_frame=960),
+    # the paper's long-rollout window: 1 sink frame + the 6 newest frames,
+    # k^R cached unrotated and re-indexed per window, frames to 960, batch 4
+    "sink": Workload("sink", batch=4, window_frames=7, sink_frames=1, last_frame=960),
 }
 
 
@@ -135,6 +139,13 @@ def grid_positions(w, first_frame, n_frames, batch=None):
     ww = np.tile(np.arange(w.grid_w), w.grid_h * n_frames)
     pos = np.stack([t, hh, ww], axis=-1).astype(np.int32)
     return torch.from_numpy(np.repeat(pos[None], B, axis=0))
+
+
+def frame_coords(w):
+    """(h, w) of token k of a latent frame, raster order: int32 [T, 2]."""
+    hh = np.repeat(np.arange(w.grid_h), w.grid_w)
+    ww = np.tile(np.arange(w.grid_w), w.grid_h)
+    return torch.from_numpy(np.stack([hh, ww], axis=-1).astype(np.int32))
 
 
 def draw_queries(w, n_tokens, seed, batch=None):

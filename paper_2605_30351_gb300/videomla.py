@@ -26,13 +26,14 @@ MLA_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 MLA_FLAG_NO_RMSNORM = 1
 MLA_FLAG_SIMT = 2
+MLA_FLAG_ROTATE_AT_USE = 4
 
 # Every symbol include/videomla.h declares.
 EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
            "mla_query_prologue_noalloc", "mla_output_projection", "mla_dense_attention_forward",
-           "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
+           "mla_window_workspace_bytes", "mla_attention_window_forward", "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
 
 
 class mla_config(ctypes.Structure):
@@ -45,6 +46,7 @@ class mla_config(ctypes.Structure):
         ("rope_theta", ctypes.c_double), ("rope_table_len", ctypes.c_int),
         ("tokens_per_frame", ctypes.c_int), ("window_frames", ctypes.c_int),
         ("batch", ctypes.c_int), ("rms_eps", ctypes.c_float), ("flags", ctypes.c_uint),
+        ("sink_frames", ctypes.c_int),
     ]
 
 
@@ -96,11 +98,15 @@ def load():
     lib.mla_output_projection.argtypes = [P(mla_config), VP, VP, I, VP, VP]
     lib.mla_query_prologue_noalloc.argtypes = [P(mla_config), VP, VP, VP, I, VP, VP, VP]
     lib.mla_dense_attention_forward.argtypes = [P(mla_config), VP, VP, VP, I, I, I, VP, VP]
+    lib.mla_window_workspace_bytes.argtypes = [P(mla_config), I]
+    lib.mla_window_workspace_bytes.restype = ctypes.c_ulonglong
+    lib.mla_attention_window_forward.argtypes = [P(mla_cache), VP, VP, VP, I, VP, VP,
+                                                 ctypes.c_ulonglong, VP, VP]
     for name in ("mla_rope_table_fill", "mla_config_check", "mla_cache_reset", "mla_cache_append",
                  "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
                  "mla_query_prologue_noalloc", "mla_output_projection",
-                 "mla_dense_attention_forward"):
+                 "mla_dense_attention_forward", "mla_attention_window_forward"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -112,14 +118,19 @@ def _check(fn, code):
 
 
 def make_config(w, flags=0):
-    """mla_config from a synth.Workload-like object."""
+    """mla_config from a synth.Workload-like object (a workload with sink
+    frames keeps k^R unrotated: the long-rollout window of App. D.4-D.5)."""
+    sink = getattr(w, "sink_frames", 0)
+    if sink:
+        flags |= MLA_FLAG_ROTATE_AT_USE
     return mla_config(
         hidden=w.hidden, heads=w.heads, head_dim=w.head_dim, d_c=w.d_c, d_r=w.d_r, d_q=w.d_q,
         rope_pairs_t=w.rope_pairs[0], rope_pairs_h=w.rope_pairs[1], rope_pairs_w=w.rope_pairs[2],
         rope_dim_t=w.rope_axis_dims[0], rope_dim_h=w.rope_axis_dims[1],
         rope_dim_w=w.rope_axis_dims[2], rope_theta=w.rope_theta,
         rope_table_len=w.rope_table_len, tokens_per_frame=w.tokens_per_frame,
-        window_frames=w.window_frames, batch=w.batch, rms_eps=w.rms_eps, flags=flags)
+        window_frames=w.window_frames, batch=w.batch, rms_eps=w.rms_eps, flags=flags,
+        sink_frames=sink)
 
 
 def mla_config_check(cfg):
@@ -203,7 +214,8 @@ def mla_cache_append(cache, x, w_dkv, gamma_kv, w_kr, pos, first_frame, n_frames
         _dev(w_dkv, bf, (cfg.d_c, cfg.hidden), "w_dkv"),
         None if gamma_kv is None else _dev(gamma_kv, bf, (cfg.d_c,), "gamma_kv"),
         _dev(w_kr, bf, (cfg.d_r, cfg.hidden), "w_kr"),
-        _dev(pos, torch.int32, (cfg.batch, n_tok, 3), "pos"),
+        None if pos is None and cfg.flags & MLA_FLAG_ROTATE_AT_USE
+        else _dev(pos, torch.int32, (cfg.batch, n_tok, 3), "pos"),
     )
     _check("mla_cache_append",
            load().mla_cache_append(ctypes.byref(cache.struct), *args, int(first_frame),
@@ -223,6 +235,32 @@ def mla_attention_forward(cache, q_c, q_r, q_pos, o_lat, stream=None):
     _check("mla_attention_forward",
            load().mla_attention_forward(ctypes.byref(cache.struct), *args, int(Nq), out,
                                         _stream_ptr(stream)))
+
+
+def mla_window_workspace_bytes(cfg, Nq):
+    return int(load().mla_window_workspace_bytes(ctypes.byref(cfg), int(Nq)))
+
+
+def mla_attention_window_forward(cache, q_c, q_r, q_pos, frame_hw, workspace, o_lat, stream=None):
+    """Attention over the assembled sink + FIFO window with window-relative
+    RoPE (App. D.4, D.5); q_pos holds absolute frames, frame_hw [T, 2] the
+    (h, w) of every token of a latent frame."""
+    cfg = cache.cfg
+    Nq = q_c.shape[1]
+    bf = torch.bfloat16
+    if not (isinstance(workspace, torch.Tensor) and workspace.is_cuda and workspace.is_contiguous()):
+        raise TypeError("workspace must be a contiguous CUDA tensor")
+    _check("mla_attention_window_forward",
+           load().mla_attention_window_forward(
+               ctypes.byref(cache.struct),
+               _dev(q_c, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "q_c"),
+               _dev(q_r, bf, (cfg.batch, Nq, cfg.heads, cfg.d_r), "q_r"),
+               _dev(q_pos, torch.int32, (cfg.batch, Nq, 3), "q_pos"), int(Nq),
+               _dev(frame_hw, torch.int32, (cfg.tokens_per_frame, 2), "frame_hw"),
+               ctypes.c_void_p(workspace.data_ptr()),
+               workspace.numel() * workspace.element_size(),
+               _dev(o_lat, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "o_lat"),
+               _stream_ptr(stream)))
 
 
 def absorbed_weight_shapes(cfg):

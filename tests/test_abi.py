@@ -32,11 +32,12 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_struct_layout_matches_header():
-    # 12 ints, a double, 4 ints, a float, an unsigned (natural C alignment)
-    assert ctypes.sizeof(V.mla_config) == 80
+    # 12 ints, a double, 4 ints, a float, an unsigned, an int, padded to 8
+    assert ctypes.sizeof(V.mla_config) == 88
     assert V.mla_config.rope_theta.offset == 48
+    assert V.mla_config.sink_frames.offset == 80
     # three pointers, a long long, the config
-    assert ctypes.sizeof(V.mla_cache) == 112
+    assert ctypes.sizeof(V.mla_cache) == 120
     assert V.mla_cache.cfg.offset == 32
 
 
@@ -56,6 +57,39 @@ def test_config_validation():
     bad = V.make_config(w)
     bad.window_frames = 0
     assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    bad = V.make_config(w)
+    bad.sink_frames = w.window_frames         # no frame slot left for the FIFO part
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    bad.sink_frames = -1
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    sink = V.make_config(synth.workload("sink"))
+    assert V.mla_config_check(sink) == V.MLA_OK
+    assert sink.sink_frames == 1 and sink.flags & V.MLA_FLAG_ROTATE_AT_USE
+
+
+def test_window_path_argument_rules():
+    """Rotate-at-use caches must go through the window entry point and vice
+    versa; the window workspace is sized for keys plus query positions."""
+    lib = V.load()
+    fake = ctypes.c_void_p(1 << 20)
+    w = synth.workload("sink")
+    cfg = V.make_config(w)
+    cache = V.mla_cache(c=fake, kr=fake, rope_table=fake, frames_written=9, cfg=cfg)
+    assert lib.mla_attention_forward(ctypes.byref(cache), fake, fake, fake, 4680, fake,
+                                     None) == V.MLA_ERR_ARG
+    need = V.mla_window_workspace_bytes(cfg, 4680)
+    keys = w.batch * w.slots * w.d_r * 2
+    assert need == (keys + 255) // 256 * 256 + w.batch * 4680 * 12
+    assert lib.mla_attention_window_forward(ctypes.byref(cache), fake, fake, fake, 4680, fake,
+                                            fake, need - 1, fake, None) == V.MLA_ERR_ARG
+    plain = V.mla_cache(c=fake, kr=fake, rope_table=fake, frames_written=21,
+                        cfg=V.make_config(synth.workload("wan")))
+    assert lib.mla_attention_window_forward(ctypes.byref(plain), fake, fake, fake, 4680, fake,
+                                            fake, need, fake, None) == V.MLA_ERR_ARG
+    # a rotate-at-use append does not need positions: NULL pos passes the
+    # host checks up to the frame-range rule
+    assert lib.mla_cache_append(ctypes.byref(cache), fake, fake, None, fake, None, 0,
+                                w.window_frames + 1, None) == V.MLA_ERR_RANGE
 
 
 def test_null_arguments_rejected_before_launch():
