@@ -502,6 +502,31 @@ def run_sweep(args, rank):
         "ms_per_chunk_layer": ms, "tflops": fl / (ms * 1e-3) / 1e12,
         "frac_of_measured_bf16_burst": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"],
         "flop_per_row_key": 4 * w.head_dim})
+    # decompress-then-dense on the d_c = 192 latent cache: expand every slot into
+    # per-head keys [W_up^K c | k] and values W_up^V c, then the dense kernel
+    s = LayerSet(base, 7300, V)
+    wt = {k: t.cuda() for k, t in synth.draw_layer_weights(base, 7301).items()}
+    kd = torch.empty(1, w.heads, w.slots, w.head_dim, dtype=torch.bfloat16, device="cuda")
+    vd = torch.empty_like(kd)
+    t_dec = time_launches(lambda: V.mla_decompress_window(s.cache, wt["w_uk"], wt["w_uv"], kd, vd,
+                                                          stream), args.steps, 2, stream)
+    t_att = time_launches(lambda: V.mla_dense_attention_forward(cfg, q, kd, vd, w.slots, o, stream),
+                          args.steps, 2, stream)
+    dn = w.head_dim - base.d_r
+    fl_dec = 2.0 * w.slots * base.d_c * w.heads * (dn + w.head_dim)
+    rows.append({
+        "layout": "mla decompress-then-dense", "d_c": base.d_c, "d_r": base.d_r,
+        "kernel": "tcgen05 (scatter GEMM + dense attention)",
+        "bytes_per_token_per_layer": 2 * (base.d_c + base.d_r),
+        "transient_bytes_per_layer": 2 * 2 * w.heads * w.head_dim * w.slots,
+        "decompress_ms": t_dec, "attention_ms": t_att, "ms_per_chunk_layer": t_dec + t_att,
+        "tflops": (fl + fl_dec) / ((t_dec + t_att) * 1e-3) / 1e12,
+        "frac_of_measured_bf16_burst": (fl + fl_dec) / ((t_dec + t_att) * 1e-3) / 1e12
+        / peaks["bf16_tflops"],
+        "flop_per_row_key": 4 * w.head_dim,
+        "decompress_flop_per_key": 2 * base.d_c * w.heads * (dn + w.head_dim)})
+    if V.mla_device_status(clear=True) != V.MLA_OK:
+        raise RuntimeError("device status set during the sweep")
     if rank != 0:
         return None
     return {"metric": "latent-size sweep: absorbed MLA attention vs dense per-head baseline",

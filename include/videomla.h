@@ -299,6 +299,24 @@ int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void
                                 const void* v, int slots, int n_valid, int Nq, void* o,
                                 void* stream);
 
+/*
+ * Decompress-then-dense: the non-absorbed way to run attention on the latent
+ * cache (Sec. 3.1 Eq. reconstruct; App. E is what it avoids). Expands every
+ * slot of the cache into per-head keys and values,
+ *     k[b][h][j] = [ W_up,h^K c_j | k_j ]     (d_nope + d_r = head_dim columns)
+ *     v[b][h][j] =   W_up,h^V c_j             (head_dim columns)
+ * so that mla_dense_attention_forward can run on them with per-head queries
+ * [q^nope_h | RoPE3D(q^R_h)] (Eq. score). All W*T slots are written.
+ *  w_uk  bf16 [heads][head_dim - d_r][d_c]    W_up^K
+ *  w_uv  bf16 [heads][head_dim][d_c]          W_up^V
+ *  k, v  bf16 [batch][heads][W*T][head_dim]   outputs (caller-owned)
+ * MLA_ERR_ARG for a cache with MLA_FLAG_ROTATE_AT_USE (its k is unrotated);
+ * MLA_ERR_UNSUPPORTED unless d_c is a multiple of 64 and head_dim - d_r a
+ * multiple of 8.
+ */
+int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* w_uv, void* k,
+                          void* v, void* stream);
+
 /* Human-readable name of a status code. */
 const char* mla_status_string(int status);
 

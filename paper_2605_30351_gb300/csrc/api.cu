@@ -291,6 +291,36 @@ int mla_attention_forward(const mla_cache* cache, const void* q_c, const void* q
                        static_cast<cudaStream_t>(stream));
 }
 
+int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* w_uv, void* k,
+                          void* v, void* stream) {
+  if (!cache) return MLA_ERR_ARG;
+  const int rc = check_config(&cache->cfg);
+  if (rc != MLA_OK) return rc;
+  const mla_config& c = cache->cfg;
+  if (rotate_at_use(c) || c.head_dim <= c.d_r) return MLA_ERR_ARG;
+  if (!cache->c || !cache->kr || !w_uk || !w_uv || !k || !v) return MLA_ERR_ARG;
+  if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(w_uk) || !aligned16(w_uv) ||
+      !aligned16(k) || !aligned16(v))
+    return MLA_ERR_ARG;
+  DecompressArgs a;
+  a.c = cache->c;
+  a.kr = cache->kr;
+  a.w_uk = w_uk;
+  a.w_uv = w_uv;
+  a.k = k;
+  a.v = v;
+  a.batch = c.batch;
+  a.slots = c.tokens_per_frame * c.window_frames;
+  a.heads = c.heads;
+  a.head_dim = c.head_dim;
+  a.d_c = c.d_c;
+  a.d_r = c.d_r;
+  a.status = device_status_ptr();
+  a.stream = static_cast<cudaStream_t>(stream);
+  if (!a.status) return fail_cuda(cudaGetLastError());
+  return launch_decompress(a);
+}
+
 unsigned long long mla_window_workspace_bytes(const mla_config* cfg, int Nq) {
   if (check_config(cfg) != MLA_OK || Nq < 1) return 0;
   return window_kr_bytes(*cfg) + static_cast<unsigned long long>(cfg->batch) * Nq * 3 * 4;

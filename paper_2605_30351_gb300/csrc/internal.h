@@ -120,6 +120,19 @@ struct WindowArgs {
   cudaStream_t stream;
 };
 
+// Decompression of the latent cache into per-head keys and values.
+struct DecompressArgs {
+  const void* c;        // bf16 [B][slots][d_c]
+  const void* kr;       // bf16 [B][slots][d_r] rotated positional keys
+  const void* w_uk;     // bf16 [H][head_dim - d_r][d_c]
+  const void* w_uv;     // bf16 [H][head_dim][d_c]
+  void* k;              // out bf16 [B][H][slots][head_dim]
+  void* v;              // out bf16 [B][H][slots][head_dim]
+  int batch, slots, heads, head_dim, d_c, d_r;
+  int* status;
+  cudaStream_t stream;
+};
+
 // Each launcher returns MLA_OK, MLA_ERR_UNSUPPORTED or MLA_ERR_CUDA.
 int launch_attention_tc(const AttnArgs& a);
 int launch_attention_simt(const AttnArgs& a);
@@ -130,6 +143,7 @@ int launch_query_prologue(const QueryArgs& a);
 int launch_output_projection(const OutProjArgs& a);
 int launch_dense_attention_tc(const DenseArgs& a);
 int launch_window_assemble(const WindowArgs& a);
+int launch_decompress(const DecompressArgs& a);
 // Device address of the fixed no-allocation scratch on the current device.
 int query_scratch_address(void** out);
 

@@ -33,7 +33,8 @@ EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
            "mla_query_prologue_noalloc", "mla_output_projection", "mla_dense_attention_forward",
-           "mla_window_workspace_bytes", "mla_attention_window_forward", "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
+           "mla_window_workspace_bytes", "mla_attention_window_forward", "mla_decompress_window",
+           "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
 
 
 class mla_config(ctypes.Structure):
@@ -98,6 +99,7 @@ def load():
     lib.mla_output_projection.argtypes = [P(mla_config), VP, VP, I, VP, VP]
     lib.mla_query_prologue_noalloc.argtypes = [P(mla_config), VP, VP, VP, I, VP, VP, VP]
     lib.mla_dense_attention_forward.argtypes = [P(mla_config), VP, VP, VP, I, I, I, VP, VP]
+    lib.mla_decompress_window.argtypes = [P(mla_cache), VP, VP, VP, VP, VP]
     lib.mla_window_workspace_bytes.argtypes = [P(mla_config), I]
     lib.mla_window_workspace_bytes.restype = ctypes.c_ulonglong
     lib.mla_attention_window_forward.argtypes = [P(mla_cache), VP, VP, VP, I, VP, VP,
@@ -106,7 +108,8 @@ def load():
                  "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
                  "mla_query_prologue_noalloc", "mla_output_projection",
-                 "mla_dense_attention_forward", "mla_attention_window_forward"):
+                 "mla_dense_attention_forward", "mla_attention_window_forward",
+                 "mla_decompress_window"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -261,6 +264,20 @@ def mla_attention_window_forward(cache, q_c, q_r, q_pos, frame_hw, workspace, o_
                workspace.numel() * workspace.element_size(),
                _dev(o_lat, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "o_lat"),
                _stream_ptr(stream)))
+
+
+def mla_decompress_window(cache, w_uk, w_uv, k, v, stream=None):
+    """Expand the latent cache into per-head keys [W_up^K c | k] and values
+    W_up^V c, both [B, H, W*T, head_dim] (the decompress-then-dense form)."""
+    cfg = cache.cfg
+    H, dh, dr, dc = cfg.heads, cfg.head_dim, cfg.d_r, cfg.d_c
+    shape = (cfg.batch, H, cache.slots, dh)
+    bf = torch.bfloat16
+    _check("mla_decompress_window",
+           load().mla_decompress_window(
+               ctypes.byref(cache.struct), _dev(w_uk, bf, (H, dh - dr, dc), "w_uk"),
+               _dev(w_uv, bf, (H, dh, dc), "w_uv"), _dev(k, bf, shape, "k"),
+               _dev(v, bf, shape, "v"), _stream_ptr(stream)))
 
 
 def absorbed_weight_shapes(cfg):

@@ -57,3 +57,101 @@ def test_dense_attention_wan_shape_sampled_rows():
     rows = np.array([0, 1, 777, 2500, 4001, w.chunk_tokens - 1])
     ref = O.dense_attention(f64(q[0, rows]), f64(k[0]), f64(v[0]), w.head_dim)
     assert_close(f64(o[0, rows]), ref, what="dense o at the Wan shape")
+
+
+# ------------------------------------------------- decompress-then-dense
+def _upload_cache(w, seed):
+    cache = V.LatentCache(V.make_config(w))
+    c, k = synth.draw_cache_rows(w, w.slots, seed)
+    cache.c.copy_(c)
+    cache.kr.copy_(k)
+    cache.frames_written = w.window_frames
+    return cache, f64(c), f64(k)
+
+
+def _decompress(w, cache, wt):
+    shape = (w.batch, w.heads, w.slots, w.head_dim)
+    k = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
+    v = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
+    V.mla_decompress_window(cache, wt["w_uk"].cuda(), wt["w_uv"].cuda(), k, v)
+    torch.cuda.synchronize()
+    return k, v
+
+
+@pytest.mark.parametrize("name,kw,slots_checked", [
+    ("tiny", dict(grid_h=10, grid_w=10, window_frames=5, batch=2), None),   # 500 slots: ragged
+    ("wan", dict(), [0, 1, 127, 128, 16001, 32759]),                        # Wan window, sampled
+])
+def test_decompress_reconstructs_per_head_keys_and_values(name, kw, slots_checked):
+    """Eq. (reconstruct): k_h = [W_up,h^K c | k], v_h = W_up,h^V c for every slot."""
+    w = synth.workload(name, **kw)
+    wt = synth.draw_layer_weights(w, seed=61)
+    cache, c, kr = _upload_cache(w, 62)
+    k, v = _decompress(w, cache, wt)
+    sl = np.arange(w.slots) if slots_checked is None else np.array(slots_checked)
+    dn = w.head_dim - w.d_r
+    k_nope = np.einsum("hec,bjc->bhje", f64(wt["w_uk"]), c[:, sl])
+    v_ref = np.einsum("hvc,bjc->bhjv", f64(wt["w_uv"]), c[:, sl])
+    kg, vg = k[:, :, sl].cpu(), v[:, :, sl].cpu()
+    assert_close(f64(kg[..., :dn]), k_nope, what="k_nope")
+    assert_close(f64(vg), v_ref, what="v")
+    # the positional part is the cached key itself, copied for every head
+    rope_bits = kg[..., dn:].view(torch.int16)
+    src = cache.kr.cpu()[:, sl].view(torch.int16)
+    for h in range(w.heads):
+        assert torch.equal(rope_bits[:, h], src)
+
+
+def test_decompress_then_dense_matches_non_absorbed_oracle():
+    """x -> GPU append -> decompress -> dense attention with per-head queries
+    [q^nope | RoPE(q^R)], against the oracle's non-absorbed forward (Sec. 3.3)."""
+    from test_gpu_parity import spec_of
+
+    w = synth.workload("tiny", grid_h=8, grid_w=10, window_frames=3, chunk_frames=1, batch=2)
+    wt = synth.draw_layer_weights(w, seed=63)
+    dev = {k: v.cuda() for k, v in wt.items()}
+    cache = V.LatentCache(V.make_config(w))
+    V.mla_cache_reset(cache)
+    T = w.tokens_per_frame
+    xs, ps = [], []
+    for f in range(4):                                   # frame 0 is evicted
+        x = synth.draw_tokens(w, T, 64 + f)
+        pos = synth.grid_positions(w, f, 1)
+        V.mla_cache_append(cache, x.cuda(), dev["w_dkv"], dev["gamma_kv"], dev["w_kr"],
+                           pos.cuda(), f, 1)
+        xs.append(x)
+        ps.append(pos)
+    k, v = _decompress(w, cache, wt)
+    w64 = {name: f64(t) for name, t in wt.items()}
+    spec = spec_of(w)
+    x_q, pos_q = xs[-1], ps[-1]
+    q = []
+    for b in range(w.batch):
+        c_q = O.rmsnorm(f64(x_q[b]) @ w64["w_dq"].T, w64["gamma_q"], w.rms_eps)
+        q_nope = np.einsum("heq,nq->nhe", w64["w_uq"], c_q)
+        q_rope = O.rope3d(np.einsum("hrq,nq->nhr", w64["w_qr"], c_q), pos_q[b].numpy()[:, None],
+                          spec)
+        q.append(np.concatenate([q_nope, q_rope], axis=-1))
+    q = synth.bf16(np.stack(q)).cuda()
+    o = torch.empty_like(q)
+    V.mla_dense_attention_forward(cache.cfg, q, k, v, cache.n_valid(), o)
+    torch.cuda.synchronize()
+    refs = []
+    for b in range(w.batch):
+        x_kv = np.concatenate([f64(xs[f][b]) for f in (1, 2, 3)])
+        pos_kv = np.concatenate([ps[f][b].numpy() for f in (1, 2, 3)])
+        refs.append(O.reference_attention(f64(x_q[b]), pos_q[b].numpy(), x_kv, pos_kv,
+                                          {n: t for n, t in w64.items() if n != "w_o"},
+                                          w.head_dim, spec, eps=w.rms_eps))
+    assert_close(f64(o), np.stack(refs), what="decompress-then-dense o")
+
+
+def test_decompress_refuses_rotate_at_use_cache():
+    w = synth.workload("tiny", window_frames=4, sink_frames=1)
+    cache = V.LatentCache(V.make_config(w))
+    wt = synth.draw_layer_weights(w, seed=65)
+    shape = (w.batch, w.heads, w.slots, w.head_dim)
+    k = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(V.MlaError) as e:
+        V.mla_decompress_window(cache, wt["w_uk"].cuda(), wt["w_uv"].cuda(), k, torch.empty_like(k))
+    assert e.value.code == V.MLA_ERR_ARG
