@@ -313,26 +313,58 @@ def run_ours(args, w, rank, world, local_rank):
     if w.layers > 1:
         e2e_steps = max(3, min(e2e_steps, 10))
 
-    def e2e_step(i):
-        for L in range(w.layers):
-            j = (i * w.layers + L) % n_e2e
-            s, h = sets[j], h_sets[j]
+    # Pipelined: each (step, layer) unit has its own device set; its inputs
+    # go up on one copy stream and its output comes back on another, so the
+    # copies of neighbouring units overlap the kernels of this one.
+    h2d_stream, d2h_stream = torch.cuda.Stream(), torch.cuda.Stream()
+    uploaded = [torch.cuda.Event() for _ in range(n_e2e)]
+    computed = [torch.cuda.Event() for _ in range(n_e2e)]
+    downloaded = [torch.cuda.Event() for _ in range(n_e2e)]
+    used = [False] * n_e2e
+
+    def upload(u):
+        j = u % n_e2e
+        s, h = sets[j], h_sets[j]
+        with torch.cuda.stream(h2d_stream):
+            if used[j]:
+                h2d_stream.wait_event(computed[j])  # the set's inputs were last read there
             s.x.copy_(h["x"], non_blocking=True)
             s.q_c.copy_(h["q_c"], non_blocking=True)
             s.q_r.copy_(h["q_r"], non_blocking=True)
             s.pos.copy_(h["pos"], non_blocking=True)
-            layer(s)
-            h["o"].copy_(s.o, non_blocking=True)
+            uploaded[j].record(h2d_stream)
 
-    for i in range(2):
-        e2e_step(i)
+    def compute_and_d2h(u):
+        j = u % n_e2e
+        s, h = sets[j], h_sets[j]
+        stream.wait_event(uploaded[j])
+        if used[j]:
+            stream.wait_event(downloaded[j])  # the set's output buffer is free again
+        layer(s)
+        computed[j].record(stream)
+        used[j] = True
+        with torch.cuda.stream(d2h_stream):
+            d2h_stream.wait_event(computed[j])
+            h["o"].copy_(s.o, non_blocking=True)
+            downloaded[j].record(d2h_stream)
+
+    def e2e_run(n_steps):
+        units = n_steps * w.layers
+        upload(0)
+        for u in range(units):
+            if u + 1 < units:
+                upload(u + 1)
+            compute_and_d2h(u)
+        stream.wait_stream(d2h_stream)
+
+    e2e_run(2)
     torch.cuda.synchronize()
     barrier(world)
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for i in range(e2e_steps):
-        e2e_step(i)
+    h2d_stream.wait_event(e0)
+    e2e_run(e2e_steps)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = allreduce_max(e0.elapsed_time(e1), world)
@@ -393,6 +425,9 @@ def run_ours(args, w, rank, world, local_rank):
             "value": whole_job_throughput(attn_fl + app_fl, e2e_ms / e2e_steps, world),
             "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": e2e_ms / e2e_steps, "steps": e2e_steps,
+            "note": "public API with pinned host buffers; every step's inputs go up and its "
+                    "latent output comes back inside the timed region, on two copy streams "
+                    "that overlap neighbouring layers' kernels",
         },
         "clocks": clk.summary(),
         "gpu_launches": (3 if w.sink_frames else 2) * w.layers * args.steps,
