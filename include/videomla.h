@@ -195,9 +195,9 @@ unsigned long long mla_window_workspace_bytes(const mla_config* cfg, int Nq);
  *     the valid slots with the rotated window keys.
  * Before any eviction local and absolute times agree. Arguments as for
  * mla_attention_forward, plus:
- *  frame_hw  int32 [tokens_per_frame][2]: (h, w) of token k of every latent
- *            frame (the latent grid is the same for all frames); each must
- *            lie in [0, rope_table_len) (device-checked)
+ *  frame_hw  int32 [tokens_per_frame][2], 8-byte aligned: (h, w) of token k
+ *            of every latent frame (the latent grid is the same for all
+ *            frames); each must lie in [0, rope_table_len) (device-checked)
  *  workspace device memory of at least mla_window_workspace_bytes(cfg, Nq)
  *            bytes, 16-byte aligned, owned by the caller (scratch)
  * A query frame the window does not hold is recorded as MLA_ERR_RANGE in

@@ -339,7 +339,7 @@ int mla_attention_window_forward(const mla_cache* cache, const void* q_c, const 
     return MLA_ERR_ARG;
   if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(q_c) || !aligned16(q_r) ||
       !aligned16(o_lat) || !aligned16(cache->rope_table) || !aligned16(workspace) ||
-      (reinterpret_cast<uintptr_t>(q_pos) & 3u) || (reinterpret_cast<uintptr_t>(frame_hw) & 3u))
+      (reinterpret_cast<uintptr_t>(q_pos) & 3u) || (reinterpret_cast<uintptr_t>(frame_hw) & 7u))
     return MLA_ERR_ARG;
   if (workspace_bytes < mla_window_workspace_bytes(&c, Nq)) return MLA_ERR_ARG;
   const long long n_valid = valid_slots(*cache);

@@ -8,9 +8,10 @@
 // slot and the queries' local positions into caller workspace; the
 // absorbed-form attention kernel then runs on them unchanged.
 //
-// One thread per (batch, slot, complex pair) reads one bf16x2 of k^R and
-// writes one bf16x2 of RoPE3D(k^R): 4 bytes in and out, coalesced along the
-// pair index. The tail of the index range handles one query token each.
+// One thread per (batch, slot, four complex pairs) reads 16 bytes of k^R and
+// writes 16 bytes of RoPE3D(k^R), coalesced along the key; each block first
+// tabulates the local time of every frame slot in shared memory. The tail of
+// the index range handles one query token each.
 #include "internal.h"
 #include "ptx_sm103.cuh"
 
@@ -44,38 +45,52 @@ __device__ __forceinline__ int checked(int v, int len, int* status) {
   return v;
 }
 
+constexpr int kMaxFrames = 1024;  // window frames whose local times a block tabulates
+
 __global__ void __launch_bounds__(kThreads)
-    window_assemble_kernel(const uint32_t* __restrict__ kr, const int* __restrict__ q_pos,
-                           const int* __restrict__ frame_hw, const float2* __restrict__ rope,
-                           uint32_t* __restrict__ kr_rot, int* __restrict__ q_local, int batch,
+    window_assemble_kernel(const uint4* __restrict__ kr, const int* __restrict__ q_pos,
+                           const int2* __restrict__ frame_hw, const float2* __restrict__ rope,
+                           uint4* __restrict__ kr_rot, int* __restrict__ q_local, int batch,
                            int nq, int slots, int n_valid, int T, int W, int S, int pairs,
                            long long fw, int rope_len, int pairs_t, int pairs_h, int* status) {
-  const long long n_key = static_cast<long long>(batch) * n_valid * pairs;
+  // local time of the frame held in each frame slot (-1: none), once per block
+  __shared__ int t_of_slot[kMaxFrames];
+  for (int j = threadIdx.x; j < W && j < kMaxFrames; j += kThreads)
+    t_of_slot[j] = static_cast<int>(local_time(frame_in_slot(j, fw, W, S), fw, W, S));
+  __syncthreads();
+  const int J = pairs / 4;  // 16-byte pieces (four complex pairs) per key
+  const long long n_key = static_cast<long long>(batch) * n_valid * J;
   const long long n_all = n_key + static_cast<long long>(batch) * nq;
   for (long long i = blockIdx.x * static_cast<long long>(kThreads) + threadIdx.x; i < n_all;
        i += static_cast<long long>(gridDim.x) * kThreads) {
     if (i < n_key) {
-      const int pr = static_cast<int>(i % pairs);
-      const long long bs = i / pairs;
+      const int c = static_cast<int>(i % J);
+      const long long bs = i / J;
       const int s = static_cast<int>(bs % n_valid);
       const int b = static_cast<int>(bs / n_valid);
-      const int k = s % T;
-      long long t = local_time(frame_in_slot(s / T, fw, W, S), fw, W, S);
+      const int fslot = s / T, k = s - fslot * T;
+      long long t = fslot < kMaxFrames ? t_of_slot[fslot]
+                                       : local_time(frame_in_slot(fslot, fw, W, S), fw, W, S);
       if (t < 0) {  // a valid slot always holds a held frame; guard regardless
         record_status(status, MLA_ERR_RANGE);
         t = 0;
       }
-      int coord;
-      if (pr < pairs_t)
-        coord = checked(static_cast<int>(t), rope_len, status);
-      else
-        coord = checked(__ldg(frame_hw + 2 * k + (pr < pairs_t + pairs_h ? 0 : 1)), rope_len,
-                        status);
-      const float2 cs = __ldg(rope + static_cast<size_t>(coord) * pairs + pr);
-      const size_t off = (static_cast<size_t>(b) * slots + s) * pairs + pr;
-      const uint32_t v = __ldg(kr + off);
-      const float x0 = bf16_lo(v), x1 = bf16_hi(v);
-      kr_rot[off] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
+      const int ct = checked(static_cast<int>(t), rope_len, status);
+      const int2 hw = __ldg(frame_hw + k);
+      const int ch = checked(hw.x, rope_len, status), cw = checked(hw.y, rope_len, status);
+      const size_t off = (static_cast<size_t>(b) * slots + s) * J + c;
+      const uint4 v = __ldg(kr + off);
+      const uint32_t in[4] = {v.x, v.y, v.z, v.w};
+      uint32_t out[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int pr = 4 * c + q;
+        const int coord = pr < pairs_t ? ct : (pr < pairs_t + pairs_h ? ch : cw);
+        const float2 cs = __ldg(rope + static_cast<size_t>(coord) * pairs + pr);
+        const float x0 = bf16_lo(in[q]), x1 = bf16_hi(in[q]);
+        out[q] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
+      }
+      kr_rot[off] = make_uint4(out[0], out[1], out[2], out[3]);
     } else {
       const long long qi = i - n_key;  // (b, n) flattened
       const int* src = q_pos + qi * 3;
@@ -96,8 +111,9 @@ __global__ void __launch_bounds__(kThreads)
 
 int launch_window_assemble(const WindowArgs& a) {
   const int pairs = a.d_r / 2;
-  const long long n_all =
-      static_cast<long long>(a.batch) * a.n_valid * pairs + static_cast<long long>(a.batch) * a.nq;
+  if (pairs % 4 != 0) return MLA_ERR_UNSUPPORTED;  // d_r is a multiple of 8 by the config rules
+  const long long n_all = static_cast<long long>(a.batch) * a.n_valid * (pairs / 4) +
+                          static_cast<long long>(a.batch) * a.nq;
   if (n_all <= 0) return MLA_OK;
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess)
@@ -105,8 +121,8 @@ int launch_window_assemble(const WindowArgs& a) {
   const long long want = (n_all + kThreads - 1) / kThreads;
   const int blocks = static_cast<int>(want < 8ll * sms ? want : 8ll * sms);
   window_assemble_kernel<<<blocks, kThreads, 0, a.stream>>>(
-      static_cast<const uint32_t*>(a.kr), a.q_pos, a.frame_hw,
-      reinterpret_cast<const float2*>(a.rope), static_cast<uint32_t*>(a.kr_rot), a.q_pos_local,
+      static_cast<const uint4*>(a.kr), a.q_pos, reinterpret_cast<const int2*>(a.frame_hw),
+      reinterpret_cast<const float2*>(a.rope), static_cast<uint4*>(a.kr_rot), a.q_pos_local,
       a.batch, a.nq, a.slots, a.n_valid, a.T, a.W, a.S, pairs, a.frames_written, a.rope_len,
       a.pairs_t, a.pairs_h, a.status);
   const cudaError_t e = cudaGetLastError();
