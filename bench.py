@@ -407,8 +407,8 @@ def run_ours(args, w, rank, world, local_rank):
             "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"],
             "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
             "peak_source": f"{peaks['source']} bf16 dense (burst)",
-            "kernel": ("window_assemble_kernel + mla_attn_tc_kernel<192,32,2> (events around both)"
-                       if w.sink_frames else "mla_attn_tc_kernel<192,32,2>"),
+            "kernel": ("window_assemble_kernel + mla_attn_tc_kernel<192,32,2,128> (events around both)"
+                       if w.sink_frames else "mla_attn_tc_kernel<192,32,2,128>"),
             "algorithmic_flops_per_launch": attn_l,
             "traffic": (profiled_traffic("attn_tc_wan_traffic.json", "attn_tc.cu")
                         if w.batch == 1 else None),

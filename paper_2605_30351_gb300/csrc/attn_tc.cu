@@ -8,7 +8,9 @@
 //     P   = exp2(S * log2(e)/sqrt(d_h) - m)        online, fp32
 //     O  += P . c                                  N = d_c (192), latent output
 // One CTA owns 128 rows (one TMEM lane each) and walks the window in blocks
-// of 128 keys:
+// of BN keys (128; 64 for (d_c, d_r) = (256, 64), where a 128-row Q tile fits
+// neither TMEM next to 128-key S and P buffers nor shared memory next to two
+// key stages):
 //   warp 0     TMA producer: [c | k] tiles into a ring of shared-memory
 //              stages (c with 128-byte swizzle, k with 64-byte swizzle).
 //              CTAs run in pairs (a cluster of two consecutive row tiles of
@@ -28,9 +30,10 @@
 //              it), writes P_j (bf16) once PV_{j-1} has read the previous P,
 //              rescales O in TMEM only when its running max grows by more
 //              than 2^8, and finally writes O / l as bf16.
-// TMEM columns: S [0,128) P [128,192) O [192,192+d_c) Q [192+d_c, +(d_c+d_r)/2).
-// When Q does not fit there (d_c = 256) it stays in shared memory (TMA-loaded
-// q_c plus the rotated q_r stored by the softmax warps) and QK reads it there.
+// TMEM columns: S [0,BN) P [BN,3BN/2) O [3BN/2,3BN/2+d_c) Q [3BN/2+d_c, +(d_c+d_r)/2).
+// When Q does not fit there (d_c = 256 with BN = 128) it stays in shared memory
+// (TMA-loaded q_c plus the rotated q_r stored by the softmax warps) and QK
+// reads it there.
 // The V operand is the first d_c columns of the same key tile read MN-major,
 // so the cache is never expanded into per-head keys or values.
 #include <cmath>
@@ -42,14 +45,15 @@ namespace vmla {
 namespace {
 
 constexpr int kBM = 128;       // rows per CTA = TMEM lanes
-constexpr int kBN = 128;       // keys per block
 constexpr int kThreads = 224;  // 7 warps
 constexpr float kRescaleLog2 = 8.0f;
 
-template <int DC, int DR>
+template <int DC, int DR, int BN>
 struct AttnShape {
+  static constexpr int kBN = BN;                   // keys per block
   static constexpr int DK = DC + DR;
   static constexpr int kTileBytes = kBN * DK * 2;  // one key stage (and the smem Q tile)
+  static constexpr int kCBox = kBN * 128;          // one [BN keys x 64 columns] box of c
   static constexpr int kKrOff = DC * kBN * 2;      // byte offset of the d_r columns in a tile
   static constexpr int kTmemS = 0;
   static constexpr int kTmemP = kBN;               // bf16 P: two values per column
@@ -60,7 +64,8 @@ struct AttnShape {
   static constexpr int kBarBytes = 256;
   static constexpr int kSmemCap = 232448;
   static constexpr int kFit = (kSmemCap - 1024 - kBarBytes - kQBytes) / kTileBytes;
-  static constexpr int kStages = kFit > 4 ? 4 : kFit;
+  static constexpr int kMaxStages = BN == 128 ? 4 : 6;
+  static constexpr int kStages = kFit > kMaxStages ? kMaxStages : kFit;
   static constexpr int kSmemBytes = 1024 + kQBytes + kTileBytes * kStages + kBarBytes;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kKrSw = DR == 32 ? kSw64 : kSw128;
@@ -68,7 +73,8 @@ struct AttnShape {
   static constexpr uint32_t kKrSbo = 8 * kKrRow;  // one 8-row swizzle atom
   static constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
   static constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, DC, false, true);
-  static_assert(kBM == kBN, "the smem Q tile and a key stage share one layout");
+  static_assert(kQinTmem || kBM == kBN, "the smem Q tile and a key stage share one layout");
+  static_assert(BN == 128 || BN == 64, "key block: 128 or 64");
   static_assert(DC % 64 == 0 && DC >= 64 && DC <= 256, "d_c: multiple of 64 up to 256");
   static_assert(DR == 32 || DR == 64, "d_r: 32 or 64");
   static_assert(kTmemO + DC <= 512, "S, P and O must fit in 512 TMEM columns");
@@ -87,12 +93,13 @@ struct AttnKParams {
   int* status;
 };
 
-template <int DC, int DR, int CL>
+template <int DC, int DR, int CL, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     mla_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_qc,
                        const __grid_constant__ CUtensorMap tm_c,
                        const __grid_constant__ CUtensorMap tm_kr, const AttnKParams p) {
-  using S = AttnShape<DC, DR>;
+  using S = AttnShape<DC, DR, BN>;
+  constexpr int kBN = S::kBN;
   constexpr int NST = S::kStages;
   constexpr uint16_t kPair = static_cast<uint16_t>((1u << CL) - 1u);  // every CTA of the cluster
   static_assert(CL == 1 || CL == 2, "clusters of one or two CTAs");
@@ -167,13 +174,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive_expect_tx(&kv_full[st], S::kTileBytes);
         if constexpr (CL == 1) {
           for (int cb = 0; cb < DC / 64; ++cb)
-            tma_load_3d(kv + cb * 16384, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
+            tma_load_3d(kv + cb * S::kCBox, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
           tma_load_3d(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b);
         } else {
           // each CTA fetches every other box once and multicasts it to both
           for (int bx = crank; bx <= DC / 64; bx += CL) {
             if (bx < DC / 64)
-              tma_load_3d_mc(kv + bx * 16384, &tm_c, &kv_full[st], bx * 64, j * kBN, b, kPair);
+              tma_load_3d_mc(kv + bx * S::kCBox, &tm_c, &kv_full[st], bx * 64, j * kBN, b, kPair);
             else
               tma_load_3d_mc(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b, kPair);
           }
@@ -214,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int cb = 0; cb < DC / 64; ++cb)
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint64_t bd = sdesc(ka + cb * 16384 + k * 32, 16, 1024, kSw128);
+            const uint64_t bd = sdesc(ka + cb * S::kCBox + k * 32, 16, 1024, kSw128);
             const uint32_t acc = (cb | k) != 0 ? 1u : 0u;
             if constexpr (S::kQinTmem)
               umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + (cb * 4 + k) * 8, bd, S::kIdescQK, acc);
@@ -255,7 +262,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int s = 0; s < kBN / 16; ++s)
           umma_ts(tmem + S::kTmemO, tmem + S::kTmemP + s * 8,
-                  sdesc(va + s * 2048, 16384, 1024, kSw128), S::kIdescPV,
+                  sdesc(va + s * 2048, S::kCBox, 1024, kSw128), S::kIdescPV,
                   (i > 0 || s > 0) ? 1u : 0u);
         if constexpr (CL == 1)
           umma_commit(&kv_empty[st]);
@@ -474,20 +481,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if constexpr (CL > 1) cluster_sync();
 }
 
-template <int DC, int DR, int CL>
+template <int DC, int DR, int CL, int BN>
 int launch_tc(const AttnArgs& a) {
-  using S = AttnShape<DC, DR>;
+  using S = AttnShape<DC, DR, BN>;
   CUtensorMap tm_qc, tm_c, tm_kr;
   const unsigned long long rows = a.rows, slots = a.slots;
   if (!encode_map_3d_bf16(&tm_qc, a.q_c, DC, rows, a.batch, DC * 2ull, rows * DC * 2ull, 64,
                           kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_3d_bf16(&tm_c, a.c, DC, a.n_valid, a.batch, DC * 2ull, slots * DC * 2ull, 64,
-                          kBN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+                          S::kBN, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_3d_bf16(&tm_kr, a.kr, DR, a.n_valid, a.batch, DR * 2ull, slots * DR * 2ull, DR,
-                          kBN,
+                          S::kBN,
                           DR == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
-  auto kern = mla_attn_tc_kernel<DC, DR, CL>;
+  auto kern = mla_attn_tc_kernel<DC, DR, CL, BN>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
   if (e != cudaSuccess) {
@@ -532,9 +539,9 @@ int launch_tc(const AttnArgs& a) {
 
 // Pairs of CTAs share every key tile through TMA multicast; a single row tile
 // per batch element runs alone.
-template <int DC, int DR>
+template <int DC, int DR, int BN = 128>
 int launch_tc_pick(const AttnArgs& a) {
-  return (a.rows + kBM - 1) / kBM >= 2 ? launch_tc<DC, DR, 2>(a) : launch_tc<DC, DR, 1>(a);
+  return (a.rows + kBM - 1) / kBM >= 2 ? launch_tc<DC, DR, 2, BN>(a) : launch_tc<DC, DR, 1, BN>(a);
 }
 
 }  // namespace
@@ -545,7 +552,7 @@ int launch_attention_tc(const AttnArgs& a) {
       case 64: return launch_tc_pick<64, 32>(a);
       case 128: return launch_tc_pick<128, 32>(a);
       case 192: return launch_tc_pick<192, 32>(a);
-      case 256: return launch_tc_pick<256, 32>(a);
+      case 256: return launch_tc_pick<256, 32>(a);  // Q in shared memory (faster than 64-key blocks)
       default: break;
     }
   } else if (a.d_r == 64) {
@@ -553,6 +560,7 @@ int launch_attention_tc(const AttnArgs& a) {
       case 64: return launch_tc_pick<64, 64>(a);
       case 128: return launch_tc_pick<128, 64>(a);
       case 192: return launch_tc_pick<192, 64>(a);
+      case 256: return launch_tc_pick<256, 64, 64>(a);  // Q in TMEM needs 64-key blocks
       default: break;
     }
   }

@@ -174,6 +174,7 @@ def test_attention_parity(case, flags):
 @pytest.mark.parametrize("d_c,d_r,pairs", [
     (64, 32, (4, 6, 6)), (128, 32, (6, 5, 5)), (256, 32, (6, 5, 5)),
     (64, 64, (12, 10, 10)), (128, 64, (12, 10, 10)), (192, 64, (12, 10, 10)),
+    (256, 64, (12, 10, 10)),
 ])
 def test_attention_latent_sweep(d_c, d_r, pairs):
     w = small(d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=(44, 42, 42) if d_r == 32
