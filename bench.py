@@ -570,6 +570,83 @@ def run_sweep(args, rank):
             "sweep": rows}
 
 
+# ------------------------------------------------------------- full layer
+def run_layer(args, w, rank):
+    """The whole attention layer per chunk (Sec. 3, App. E): query prologue
+    (x -> c^Q -> RMSNorm -> [q_c | q_r], absorbed weights), cache append,
+    latent attention and output projection y = sum_h B_h o_lat,h; each phase
+    timed with CUDA events, inputs rotating over layer sets larger than L2."""
+    from paper_2605_30351_gb300 import videomla as V
+
+    V.load()
+    stream = torch.cuda.current_stream()
+    nq = w.chunk_tokens
+    sets = []
+    for i in range(N_SETS):
+        s = LayerSet(w, 1200 + 17 * i, V)
+        wt = {k: t.cuda() for k, t in synth.draw_layer_weights(w, 1200 + 17 * i).items()}
+        cfg = s.cache.cfg
+        s.w_dq = wt["w_dq"]
+        s.w_qcat, s.w_b = V.mla_absorb_weights(cfg, wt["w_uq"], wt["w_uk"], wt["w_qr"],
+                                               wt["gamma_q"], wt["w_uv"], wt["w_o"])
+        s.ws_q = torch.empty(V.mla_query_workspace_bytes(cfg, nq), dtype=torch.uint8, device="cuda")
+        s.y = torch.empty(w.batch, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
+        sets.append(s)
+
+    def layer(s, ev=None):
+        cfg = s.cache.cfg
+        if ev is not None:
+            ev[0].record(stream)
+        V.mla_query_prologue(cfg, s.x, s.w_dq, s.w_qcat, s.ws_q, s.q_c, s.q_r, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        V.mla_cache_append(s.cache, s.x, s.w_dkv, s.gamma, s.w_kr, None if s.window else s.pos,
+                           s.first, w.chunk_frames, stream)
+        if ev is not None:
+            ev[2].record(stream)
+        if s.window:
+            V.mla_attention_window_forward(s.cache, s.q_c, s.q_r, s.pos, s.hw, s.ws, s.o, stream)
+        else:
+            V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
+        if ev is not None:
+            ev[3].record(stream)
+        V.mla_output_projection(cfg, s.o, s.w_b, s.y, stream)
+        if ev is not None:
+            ev[4].record(stream)
+
+    for i in range(max(3, args.warmup)):
+        layer(sets[i % N_SETS])
+    torch.cuda.synchronize()
+    steps = max(1, args.steps)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    for i in range(steps):
+        layer(sets[i % N_SETS], evs[i])
+    torch.cuda.synchronize()
+    if V.mla_device_status(clear=True) != V.MLA_OK:
+        raise RuntimeError("device status set during the layer timing")
+    med = [float(np.median([e[k].elapsed_time(e[k + 1]) for e in evs])) for k in range(4)]
+    total = float(np.median([e[0].elapsed_time(e[4]) for e in evs]))
+    rows = w.batch * nq
+    attn_fl, app_fl = flops_per_layer(w)
+    pro_fl = 2.0 * rows * w.hidden * w.d_q + 2.0 * rows * w.d_q * w.heads * (w.d_c + w.d_r)
+    out_fl = 2.0 * rows * w.heads * w.d_c * w.hidden
+    peaks = load_peaks()
+    phases = {}
+    for name, ms, fl in (("query_prologue", med[0], pro_fl), ("append", med[1], app_fl),
+                         ("attention", med[2], attn_fl), ("output_projection", med[3], out_fl)):
+        phases[name] = {"ms": ms, "flop": fl, "tflops": fl / (ms * 1e-3) / 1e12,
+                        "frac_of_measured_bf16_burst": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"]}
+    if rank != 0:
+        return None
+    fl_all = pro_fl + app_fl + attn_fl + out_fl
+    return {"metric": "full attention layer per chunk: prologue, append, attention, output projection",
+            "value": fl_all / (total * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_layer": total,
+            "higher_is_better": True, "data": "synthetic", "dtype": "bf16", "steps": steps,
+            "config": {"workload": workload_desc(w) + "; step = the whole layer",
+                       "l2": f"{N_SETS} rotating layer sets"},
+            "phases": phases, "gpu_launches_per_layer": 5 + (1 if w.sink_frames else 0)}
+
+
 # ------------------------------------------------------ memory-cap batch sweep
 B200_USABLE_GB = 180.0  # HBM of the B200 the paper's batch-scaling figure ran on
 
@@ -743,9 +820,10 @@ def main():
     ap.add_argument("--workload", default="wan")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweep", choices=["dc", "memcap"], default=None,
+    ap.add_argument("--sweep", choices=["dc", "memcap", "layer"], default=None,
                     help="dc: latent-size sweep next to the dense baseline; memcap: maximum "
-                         "batch under --mem-budget-gb (one JSON line each)")
+                         "batch under --mem-budget-gb; layer: the whole attention layer by "
+                         "phase (one JSON line each)")
     ap.add_argument("--mem-budget-gb", type=float, default=B200_USABLE_GB)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
@@ -761,6 +839,8 @@ def main():
         out = run_sweep(args, rank)
     elif args.sweep == "memcap":
         out = run_memcap(args, rank)
+    elif args.sweep == "layer":
+        out = run_layer(args, w, rank)
     elif args.impl == "reference":
         out = run_reference(args, w, rank)
     else:

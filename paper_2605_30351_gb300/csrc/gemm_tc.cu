@@ -28,14 +28,14 @@ constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kThreads = 192;
 
-template <int BN>
+template <int BN, int MAXST>
 struct GemmShape {
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBarBytes = 256;
   static constexpr int kFit = (232448 - 1024 - kBarBytes) / kStageBytes;
-  static constexpr int kStages = kFit > 6 ? 6 : kFit;
+  static constexpr int kStages = kFit > MAXST ? MAXST : kFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
   static constexpr int kOutStride = BN * 2 + 16;  // staged bf16 row + 16 bytes (bank spread)
   static constexpr uint32_t kTmemCols = BN <= 128 ? 128 : 256;
@@ -56,11 +56,11 @@ struct GemmKParams {
 
 enum { kStore = 0, kStoreSq = 1, kRowScale = 2 };
 
-template <int BN, int EPI>
+template <int BN, int EPI, int MAXST>
 __global__ void __launch_bounds__(kThreads, 1)
     mla_gemm_tc_kernel(const __grid_constant__ CUtensorMap tm_a,
                        const __grid_constant__ CUtensorMap tm_b, const GemmKParams p) {
-  using S = GemmShape<BN>;
+  using S = GemmShape<BN, MAXST>;
   constexpr int NST = S::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_smem_1024(smem_raw);
@@ -205,16 +205,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, int MAXST = 6>
 int launch_gemm(const void* a, const void* b, int M, int N, int K, GemmKParams kp,
                 cudaStream_t stream) {
-  using S = GemmShape<BN>;
+  using S = GemmShape<BN, MAXST>;
   if (K % kBK != 0 || N % 8 != 0) return MLA_ERR_UNSUPPORTED;
   CUtensorMap tm_a, tm_b;
   if (!encode_map_2d_bf16(&tm_a, a, K, M, K * 2ull, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_b, b, K, N, K * 2ull, kBK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
-  auto kern = mla_gemm_tc_kernel<BN, EPI>;
+  auto kern = mla_gemm_tc_kernel<BN, EPI, MAXST>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
   if (e != cudaSuccess) {
@@ -321,8 +321,10 @@ int launch_query_prologue(const QueryArgs& a) {
   k2.sq_dim = static_cast<float>(a.d_q);
   k2.eps = a.eps;
   k2.status = a.status;
-  return launch_gemm<256, kRowScale>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r), a.d_q,
-                                     k2, a.stream);
+  // two-stage ring: two CTAs per SM overlap one tile's epilogue with the next
+  // one's loads (measured 48 vs 51 us at one Wan chunk, 138 vs 164 us at four)
+  return launch_gemm<256, kRowScale, 2>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
+                                        a.d_q, k2, a.stream);
 }
 
 // ---- fixed scratch for mla_query_prologue_noalloc ----
@@ -365,8 +367,18 @@ int launch_output_projection(const OutProjArgs& a) {
   k.c = static_cast<__nv_bfloat16*>(a.y);
   k.ldc = a.hidden;
   k.status = a.status;
-  return launch_gemm<256, kStore>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
-                                  a.stream);
+  // Two CTAs per SM (two-stage ring). 192-wide tiles when 256-wide ones would
+  // leave the GPU less than two CTAs per SM (one Wan chunk: 29 vs 35 us);
+  // 256-wide otherwise (four chunks: 100 vs 119 us).
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long ctas256 = static_cast<long long>((a.rows + kBM - 1) / kBM) * ((a.hidden + 255) / 256);
+  if (ctas256 < 2ll * sms && a.hidden % 192 == 0)
+    return launch_gemm<192, kStore, 2>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
+                                       a.stream);
+  return launch_gemm<256, kStore, 2>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
+                                     a.stream);
 }
 
 }  // namespace vmla

@@ -114,3 +114,25 @@ def test_full_layer_output_matches_non_absorbed_oracle():
                                           w.head_dim, spec_of(w), eps=w.rms_eps)
         refs.append(y_ref)
     assert_close(f64(y), np.stack(refs), what="layer output y")
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+def test_output_projection_at_wan_size(batch):
+    """y = o_lat W_B^T at one and four Wan chunks (the two tile widths the
+    launcher picks between), checked on sampled rows in float64."""
+    w = synth.workload("wan", batch=batch)
+    wt = synth.draw_layer_weights(w, seed=95)
+    dev = {k: v.cuda() for k, v in wt.items()}
+    cfg = V.make_config(w)
+    _w_qcat, w_b = V.mla_absorb_weights(cfg, dev["w_uq"], dev["w_uk"], dev["w_qr"], dev["gamma_q"],
+                                        dev["w_uv"], dev["w_o"])
+    g = torch.Generator(device="cuda").manual_seed(96)
+    o_lat = torch.randn(batch, w.chunk_tokens, w.heads, w.d_c, device="cuda", generator=g)
+    o_lat = o_lat.to(torch.bfloat16)
+    y = torch.empty(batch, w.chunk_tokens, w.hidden, dtype=torch.bfloat16, device="cuda")
+    V.mla_output_projection(cfg, o_lat, w_b, y)
+    torch.cuda.synchronize()
+    rows = np.array([0, 1, 127, 128, 2999, w.chunk_tokens - 1])
+    flat = f64(o_lat).reshape(batch, w.chunk_tokens, -1)[:, rows]
+    ref = flat @ f64(w_b).T
+    assert_close(f64(y)[:, rows], ref, what=f"y, batch {batch}")
