@@ -317,6 +317,17 @@ int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void
 int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* w_uv, void* k,
                           void* v, void* stream);
 
+/*
+ * Self-test of the bounded device waits that guard every mbarrier wait in the
+ * tensor-core kernels (a device wait never hangs: after its limit it records
+ * MLA_ERR_TIMEOUT in the device status word and the kernel returns). Launches
+ * one thread that waits, through the same code, on a barrier nothing arrives
+ * on, for limit_ns nanoseconds (1 ns .. 2 s); afterwards mla_device_status
+ * reports MLA_ERR_TIMEOUT and the context remains usable. MLA_ERR_ARG for a
+ * limit outside that range.
+ */
+int mla_selftest_bounded_wait(unsigned long long limit_ns, void* stream);
+
 /* Human-readable name of a status code. */
 const char* mla_status_string(int status);
 

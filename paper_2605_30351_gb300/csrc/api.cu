@@ -528,6 +528,13 @@ int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void
   return launch_dense_attention_tc(a);
 }
 
+int mla_selftest_bounded_wait(unsigned long long limit_ns, void* stream) {
+  if (limit_ns == 0 || limit_ns > 2000000000ull) return MLA_ERR_ARG;
+  int* st = device_status_ptr();
+  if (!st) return fail_cuda(cudaGetLastError());
+  return launch_wait_selftest(limit_ns, st, static_cast<cudaStream_t>(stream));
+}
+
 const char* mla_status_string(int status) {
   switch (status) {
     case MLA_OK: return "ok";

@@ -144,6 +144,7 @@ int launch_output_projection(const OutProjArgs& a);
 int launch_dense_attention_tc(const DenseArgs& a);
 int launch_window_assemble(const WindowArgs& a);
 int launch_decompress(const DecompressArgs& a);
+int launch_wait_selftest(unsigned long long limit_ns, int* status, cudaStream_t stream);
 // Device address of the fixed no-allocation scratch on the current device.
 int query_scratch_address(void** out);
 

@@ -34,7 +34,7 @@ EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
            "mla_query_prologue_noalloc", "mla_output_projection", "mla_dense_attention_forward",
            "mla_window_workspace_bytes", "mla_attention_window_forward", "mla_decompress_window",
-           "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
+           "mla_selftest_bounded_wait", "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
 
 
 class mla_config(ctypes.Structure):
@@ -100,6 +100,7 @@ def load():
     lib.mla_query_prologue_noalloc.argtypes = [P(mla_config), VP, VP, VP, I, VP, VP, VP]
     lib.mla_dense_attention_forward.argtypes = [P(mla_config), VP, VP, VP, I, I, I, VP, VP]
     lib.mla_decompress_window.argtypes = [P(mla_cache), VP, VP, VP, VP, VP]
+    lib.mla_selftest_bounded_wait.argtypes = [ctypes.c_ulonglong, VP]
     lib.mla_window_workspace_bytes.argtypes = [P(mla_config), I]
     lib.mla_window_workspace_bytes.restype = ctypes.c_ulonglong
     lib.mla_attention_window_forward.argtypes = [P(mla_cache), VP, VP, VP, I, VP, VP,
@@ -109,7 +110,7 @@ def load():
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
                  "mla_query_prologue_noalloc", "mla_output_projection",
                  "mla_dense_attention_forward", "mla_attention_window_forward",
-                 "mla_decompress_window"):
+                 "mla_decompress_window", "mla_selftest_bounded_wait"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -361,6 +362,12 @@ def mla_dense_attention_forward(cfg, q, k, v, n_valid, o, stream=None):
                _dev(k, bf, (B, H, slots, dh), "k"), _dev(v, bf, (B, H, slots, dh), "v"),
                int(slots), int(n_valid), int(Nq), _dev(o, bf, (B, Nq, H, dh), "o"),
                _stream_ptr(stream)))
+
+
+def mla_selftest_bounded_wait(limit_ns, stream=None):
+    """Make one bounded device wait run out (nothing arrives on its barrier)."""
+    _check("mla_selftest_bounded_wait",
+           load().mla_selftest_bounded_wait(int(limit_ns), _stream_ptr(stream)))
 
 
 def mla_device_status(clear=True):

@@ -111,6 +111,9 @@ def test_null_arguments_rejected_before_launch():
     assert lib.mla_cache_append(ctypes.byref(cache), odd, fake, None, fake, fake, 0, 1,
                                 None) == V.MLA_ERR_ARG
     assert lib.mla_status_string(V.MLA_ERR_RANGE).decode().startswith("frame count")
+    # the wait self-test checks its limit before launching anything
+    assert lib.mla_selftest_bounded_wait(0, None) == V.MLA_ERR_ARG
+    assert lib.mla_selftest_bounded_wait(3_000_000_000, None) == V.MLA_ERR_ARG
 
 
 @pytest.mark.parametrize("name", ["tiny", "wan"])
