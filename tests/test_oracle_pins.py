@@ -407,3 +407,21 @@ def test_dense_attention_is_sdpa():
     q, k, v = rng.standard_normal((6, 3, 8)), rng.standard_normal((3, 10, 8)), rng.standard_normal((3, 10, 8))
     ref = _sdpa(q.transpose(1, 0, 2), k, v).transpose(1, 0, 2)
     np.testing.assert_allclose(O.dense_attention(q, k, v, 8), ref, rtol=1e-12, atol=1e-12)
+
+
+def test_flop_count_matches_numpy_contraction_count():
+    """latent_attention_flops against NumPy's own operation count of the three
+    contractions latent_attention performs (scores over c and over k, then
+    P times c): two FLOPs per multiply-add of each einsum."""
+    import re
+
+    def naive(spec, *shapes):
+        info = np.einsum_path(spec, *[np.zeros(s) for s in shapes], optimize="greedy")[1]
+        return float(re.search(r"Naive FLOP count:\s*([0-9.e+]+)", info).group(1))
+
+    for nq, H, nk, dc, dr in [(3, 2, 7, 5, 4), (4, 3, 11, 8, 2), (2, 1, 1, 6, 0)]:
+        got = O.latent_attention_flops(nq * H, nk, dc, dr)
+        want = naive("nhc,jc->nhj", (nq, H, dc), (nk, dc)) + naive("nhj,jc->nhc", (nq, H, nk), (nk, dc))
+        if dr:
+            want += naive("nhr,jr->nhj", (nq, H, dr), (nk, dr))
+        assert got == want, (got, want)
