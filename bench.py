@@ -570,6 +570,57 @@ def run_sweep(args, rank):
             "sweep": rows}
 
 
+# ------------------------------------------------------------- crossover
+def run_crossover(args, rank):
+    """Absorbed attention (App. E) against decompress-then-dense (Eq.
+    reconstruct, then per-head attention) as the query chunk grows from one
+    latent frame to twelve, on the same 21-frame Wan window: the per-key cost
+    of decompressing is paid once per window, the absorbed form's extra cost
+    per (query, key)."""
+    from paper_2605_30351_gb300 import videomla as V
+
+    V.load()
+    stream = torch.cuda.current_stream()
+    peaks = load_peaks()
+    rows = []
+    for frames in (1, 2, 3, 6, 12):
+        w = synth.workload("wan", chunk_frames=frames)
+        nq = w.chunk_tokens
+        s = LayerSet(w, 7400 + frames, V)
+        wt = {k: t.cuda() for k, t in synth.draw_layer_weights(w, 7401).items()}
+        t_abs = time_launches(lambda: V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o,
+                                                              stream), args.steps, 2, stream)
+        cfg = s.cache.cfg
+        kd = torch.empty(1, w.heads, w.slots, w.head_dim, dtype=torch.bfloat16, device="cuda")
+        vd = torch.empty_like(kd)
+        g = torch.Generator(device="cuda").manual_seed(frames)
+        q = torch.randn(1, nq, w.heads, w.head_dim, device="cuda", generator=g).to(torch.bfloat16)
+        o = torch.empty_like(q)
+        t_dec = time_launches(lambda: V.mla_decompress_window(s.cache, wt["w_uk"], wt["w_uv"], kd,
+                                                              vd, stream), args.steps, 2, stream)
+        t_den = time_launches(lambda: V.mla_dense_attention_forward(cfg, q, kd, vd, w.slots, o,
+                                                                    stream), args.steps, 2, stream)
+        fl_abs = flops_per_layer(w)[0]
+        rows.append({"query_frames": frames, "query_tokens": nq, "keys": w.slots,
+                     "absorbed_ms": t_abs,
+                     "absorbed_tflops": fl_abs / (t_abs * 1e-3) / 1e12,
+                     "decompress_ms": t_dec, "dense_attention_ms": t_den,
+                     "decompress_then_dense_ms": t_dec + t_den,
+                     "absorbed_over_decompressed": t_abs / (t_dec + t_den)})
+        del s, kd, vd, q, o
+        torch.cuda.empty_cache()
+    if V.mla_device_status(clear=True) != V.MLA_OK:
+        raise RuntimeError("device status set during the crossover sweep")
+    if rank != 0:
+        return None
+    return {"metric": "absorbed MLA attention vs decompress-then-dense, by query-chunk size",
+            "unit": "ms per chunk per layer", "data": "synthetic", "dtype": "bf16",
+            "peak_bf16_tflops": peaks["bf16_tflops"],
+            "config": {"workload": "Wan2.1-1.3B layer: 21-frame window (32,760 keys), 12 heads, "
+                                   "d_c=192, d_r=32, batch 1; query chunk of 1..12 latent frames"},
+            "crossover": rows}
+
+
 # ------------------------------------------------------------- full layer
 def run_layer(args, w, rank):
     """The whole attention layer per chunk (Sec. 3, App. E): query prologue
@@ -820,10 +871,11 @@ def main():
     ap.add_argument("--workload", default="wan")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweep", choices=["dc", "memcap", "layer"], default=None,
+    ap.add_argument("--sweep", choices=["dc", "memcap", "layer", "crossover"], default=None,
                     help="dc: latent-size sweep next to the dense baseline; memcap: maximum "
                          "batch under --mem-budget-gb; layer: the whole attention layer by "
-                         "phase (one JSON line each)")
+                         "phase; crossover: absorbed vs decompress-then-dense by chunk size "
+                         "(one JSON line each)")
     ap.add_argument("--mem-budget-gb", type=float, default=B200_USABLE_GB)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
@@ -841,6 +893,8 @@ def main():
         out = run_memcap(args, rank)
     elif args.sweep == "layer":
         out = run_layer(args, w, rank)
+    elif args.sweep == "crossover":
+        out = run_crossover(args, rank)
     elif args.impl == "reference":
         out = run_reference(args, w, rank)
     else:
