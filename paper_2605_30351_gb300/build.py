@@ -41,19 +41,30 @@ def _stale(lib, deps):
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(verbose=False, force=False, extra_flags=()):
-    """Compile and link; returns the path of the library."""
+DEBUG_LIB_PATH = os.path.join(PKG, "libvideomla_debug.so")
+DEBUG_BUILD_DIR = os.path.join(PKG, "_build_debug")
+
+
+def build(verbose=False, force=False, extra_flags=(), debug=False):
+    """Compile and link; returns the path of the library. debug=True builds
+    libvideomla_debug.so with the device-side index checks switched on
+    (-DVMLA_DEBUG_CHECKS=1: a computed index out of range records
+    MLA_ERR_RANGE in the device status word and skips the access)."""
     nvcc = _nvcc()
     srcs = sources()
     deps = srcs + [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     deps.append(os.path.join(INCLUDE, "videomla.h"))
     deps.append(os.path.abspath(__file__))
-    if not force and not _stale(LIB_PATH, deps):
-        return LIB_PATH
-    os.makedirs(BUILD_DIR, exist_ok=True)
+    lib_path = DEBUG_LIB_PATH if debug else LIB_PATH
+    build_dir = DEBUG_BUILD_DIR if debug else BUILD_DIR
+    if debug:
+        extra_flags = tuple(extra_flags) + ("-DVMLA_DEBUG_CHECKS=1",)
+    if not force and not _stale(lib_path, deps):
+        return lib_path
+    os.makedirs(build_dir, exist_ok=True)
 
     def compile_one(src):
-        obj = os.path.join(BUILD_DIR, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
         cmd = [nvcc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -64,14 +75,14 @@ def build(verbose=False, force=False, extra_flags=()):
 
     with cf.ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB_PATH + ".tmp"
+    tmp = lib_path + ".tmp"
     cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
-    print(build(verbose=True, force="--force" in sys.argv))
+    print(build(verbose=True, force="--force" in sys.argv, debug="--debug" in sys.argv))

@@ -181,7 +181,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
       const long long f = p.first_frame + n / p.T;
-      slot_of[r] = row_ok ? frame_base_slot(f, p.T, p.W, p.S) + n % p.T : -1;
+      const long long slot = frame_base_slot(f, p.T, p.W, p.S) + n % p.T;
+      slot_of[r] = row_ok && debug_in_range(slot, 0, p.slots, p.status) ? slot : -1;
       uint8_t* srow = stage_out + r * S::kOutStride;
       // pass 2: gamma * c / rms -> bf16
 #pragma unroll 1

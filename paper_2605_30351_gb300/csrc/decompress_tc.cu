@@ -269,7 +269,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 4
       for (int q = et; q < kBM * chunks; q += kEpiThreads) {
         const long long rb = row_base[row];
-        if (rb >= 0)
+        if (rb >= 0 && debug_in_range(rb + col_off[ch], 0,
+                                      static_cast<long long>(p.M) * p.heads * p.head_dim - 7,
+                                      p.status))
           *reinterpret_cast<uint4*>(out + rb + col_off[ch]) =
               *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
         row += drow;
@@ -285,8 +287,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int u = et + kEpiThreads * k, row = u / kr_chunks;
           if (u < kBM * kr_chunks && row_base[row] >= 0)
             for (int a = 0; a < n_heads; ++a)
-              *reinterpret_cast<uint4*>(out + row_base[row] + head_off[a] + 8 * (u % kr_chunks)) =
-                  krv[k];
+              if (debug_in_range(row_base[row] + head_off[a] + 8 * (u % kr_chunks), 0,
+                                 static_cast<long long>(p.M) * p.heads * p.head_dim - 7, p.status))
+                *reinterpret_cast<uint4*>(out + row_base[row] + head_off[a] + 8 * (u % kr_chunks)) =
+                    krv[k];
         }
       }
       epilogue_sync();  // staging free for the next tile

@@ -28,6 +28,26 @@ __device__ __forceinline__ void record_status(int* status, int code) {
   if (status) atomicCAS(status, MLA_OK, code);
 }
 
+// Debug builds (-DVMLA_DEBUG_CHECKS=1, build(debug=True)) verify computed
+// indices (ring slots, window frame slots, scattered head offsets) before
+// they address memory: an index outside [lo, hi) records MLA_ERR_RANGE and
+// the access is skipped. Release builds compile the check away.
+#ifndef VMLA_DEBUG_CHECKS
+#define VMLA_DEBUG_CHECKS 0
+#endif
+__device__ __forceinline__ bool debug_in_range(long long v, long long lo, long long hi,
+                                               int* status) {
+#if VMLA_DEBUG_CHECKS
+  if (v < lo || v >= hi) {
+    record_status(status, MLA_ERR_RANGE);
+    return false;
+  }
+#else
+  (void)v; (void)lo; (void)hi; (void)status;
+#endif
+  return true;
+}
+
 // ----------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)

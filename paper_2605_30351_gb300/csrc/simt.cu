@@ -56,6 +56,7 @@ __global__ void append_simt_kernel(const __nv_bfloat16* __restrict__ x,
   const float inv = use_rmsnorm ? rsqrtf(red[0] / d_c + eps) : 1.f;
   const long long f = first_frame + n / T;
   const long long slot = frame_base_slot(f, T, W, S) + n % T;
+  if (!debug_in_range(slot, 0, slots, status)) return;
   __nv_bfloat16* cd = c + (static_cast<size_t>(b) * slots + slot) * d_c;
   for (int col = threadIdx.x; col < d_c; col += blockDim.x) {
     const float g = gamma ? __bfloat162float(gamma[col]) : 1.f;

@@ -69,6 +69,7 @@ __global__ void __launch_bounds__(kThreads)
       const int s = static_cast<int>(bs % n_valid);
       const int b = static_cast<int>(bs / n_valid);
       const int fslot = s / T, k = s - fslot * T;
+      if (!debug_in_range(fslot, 0, W, status)) continue;
       long long t = fslot < kMaxFrames ? t_of_slot[fslot]
                                        : local_time(frame_in_slot(fslot, fw, W, S), fw, W, S);
       if (t < 0) {  // a valid slot always holds a held frame; guard regardless

@@ -1,0 +1,67 @@
+"""Helper run in a subprocess by test_gpu_debug_build.py: loads the library
+named on the command line (release or debug build), runs a fixed set of
+calls (append + attention on the 21-frame ring, the sink window, the
+decompression, the query prologue and output projection) on seeded inputs
+and saves every output plus the device status word."""
+
+import os
+import sys
+
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+from paper_2605_30351_gb300 import synth  # noqa: E402
+from paper_2605_30351_gb300 import videomla as V  # noqa: E402
+
+
+def main(lib_path, out_path):
+    V.LIB_PATH = lib_path
+    V._lib = None
+    V.load()
+    V.mla_device_status(clear=True)
+    out = {}
+    for sink in (0, 1):
+        w = synth.workload("tiny", grid_h=10, grid_w=10, window_frames=4, sink_frames=sink, batch=2)
+        wt = {k: t.cuda() for k, t in synth.draw_layer_weights(w, 31).items()}
+        cfg = V.make_config(w)
+        cache = V.LatentCache(cfg)
+        V.mla_cache_reset(cache)
+        T = w.tokens_per_frame
+        for f in range(7):
+            x = synth.draw_tokens(w, T, 40 + f).cuda()
+            pos = None if sink else synth.grid_positions(w, f, 1).cuda()
+            V.mla_cache_append(cache, x, wt["w_dkv"], wt["gamma_kv"], wt["w_kr"], pos, f, 1)
+        q_c, q_r = synth.draw_queries(w, T, 50)
+        q_pos = synth.grid_positions(w, 6, 1).cuda()
+        o = torch.empty(w.batch, T, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+        if sink:
+            ws = torch.empty(V.mla_window_workspace_bytes(cfg, T), dtype=torch.uint8, device="cuda")
+            V.mla_attention_window_forward(cache, q_c.cuda(), q_r.cuda(), q_pos,
+                                           synth.frame_coords(w).cuda(), ws, o)
+        else:
+            V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos, o)
+            k = torch.empty(w.batch, w.heads, w.slots, w.head_dim, dtype=torch.bfloat16,
+                            device="cuda")
+            v = torch.empty_like(k)
+            V.mla_decompress_window(cache, wt["w_uk"], wt["w_uv"], k, v)
+            out["k"], out["v"] = k.cpu(), v.cpu()
+            w_qcat, w_b = V.mla_absorb_weights(cfg, wt["w_uq"], wt["w_uk"], wt["w_qr"],
+                                               wt["gamma_q"], wt["w_uv"], wt["w_o"])
+            x = synth.draw_tokens(w, T, 60).cuda()
+            wsq = torch.empty(V.mla_query_workspace_bytes(cfg, T), dtype=torch.uint8, device="cuda")
+            qc2 = torch.empty(w.batch, T, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+            qr2 = torch.empty(w.batch, T, w.heads, w.d_r, dtype=torch.bfloat16, device="cuda")
+            V.mla_query_prologue(cfg, x, wt["w_dq"], w_qcat, wsq, qc2, qr2)
+            y = torch.empty(w.batch, T, w.hidden, dtype=torch.bfloat16, device="cuda")
+            V.mla_output_projection(cfg, o, w_b, y)
+            out["q_c"], out["q_r"], out["y"] = qc2.cpu(), qr2.cpu(), y.cpu()
+        torch.cuda.synchronize()
+        out[f"c{sink}"], out[f"kr{sink}"], out[f"o{sink}"] = cache.c.cpu(), cache.kr.cpu(), o.cpu()
+    out["status"] = V.mla_device_status(clear=True)
+    torch.save(out, out_path)
+
+
+if __name__ == "__main__":
+    main(sys.argv[1], sys.argv[2])
