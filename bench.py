@@ -3,11 +3,17 @@ attention at the Wan2.1-1.3B shape (4680-query chunk, 32760-key window,
 12 heads, d_c = 192, d_r = 32, batch 1), through the C ABI.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload wan|wan30|rollout|sink]
+                  [--sweep dc|memcap|layer|crossover]
 
 One step = mla_cache_append of the current 3-frame chunk + mla_attention_forward
-of that chunk against the full 21-frame window (one layer, one denoising step).
-Prints one JSON line (rank 0). Multi-GPU runs are independent replicas
-(weak scaling): the path has no exchange step.
+of that chunk against the full 21-frame window (one layer, one denoising step;
+30 layers for wan30; batch 4 for rollout and sink, sink using the 1 + 6 frame
+window with rotate-at-use RoPE). Prints one JSON line (rank 0). Multi-GPU runs
+are independent replicas (weak scaling): the path has no exchange step. The
+--sweep modes print one JSON line each on one GPU: the latent-size sweep next
+to the dense baseline, the memory-cap batch sweep, the whole layer by phase,
+and absorbed vs decompress-then-dense by query-chunk size.
 """
 
 import argparse
