@@ -699,7 +699,9 @@ def run_layer(args, w, rank):
     return {"metric": "full attention layer per chunk: prologue, append, attention, output projection",
             "value": fl_all / (total * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_layer": total,
             "higher_is_better": True, "data": "synthetic", "dtype": "bf16", "steps": steps,
-            "config": {"workload": workload_desc(w) + "; step = the whole layer",
+            "config": {"workload": workload_desc(w).replace(
+                "step = cache append + attention", "step = query prologue + cache append + "
+                "attention + output projection"),
                        "l2": f"{N_SETS} rotating layer sets"},
             "phases": phases, "gpu_launches_per_layer": 5 + (1 if w.sink_frames else 0)}
 
