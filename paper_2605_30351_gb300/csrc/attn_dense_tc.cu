@@ -238,13 +238,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < kBN; ++c)
           if (c >= valid) sv[c] = -INFINITY;
       }
+      // three-input max: two new scores per instruction
       float m8[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) m8[i] = sv[i];
 #pragma unroll
-      for (int c = 8; c < kBN; c += 8)
+      for (int c = 8; c + 16 <= kBN; c += 16)
 #pragma unroll
-        for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[c + i]);
+        for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], sv[c + i], sv[c + 8 + i]);
+      if constexpr ((kBN - 8) % 16 != 0) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[kBN - 8 + i]);
+      }
       const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                              fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       const float m_blk = mx * p.scale_log2;
@@ -259,18 +264,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       l_run *= alpha;
       const float neg_m = -m_run;
-      float l8[8];
+      // scale-and-shift and the row sum two scores per instruction (paired
+      // fp32: the same IEEE roundings as the scalar forms, same 8 sum chains)
+      const uint64_t scale2 = f32x2_pack(p.scale_log2, p.scale_log2);
+      const uint64_t negm2 = f32x2_pack(neg_m, neg_m);
+      uint64_t l4[4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) l8[i] = 0.f;
+      for (int i = 0; i < 4; ++i) l4[i] = 0ull;
       uint32_t pk[kBN / 2];
 #pragma unroll
       for (int i = 0; i < kBN / 2; ++i) {
-        const float p0 = ex2_approx(fmaf(sv[2 * i], p.scale_log2, neg_m));
-        const float p1 = ex2_approx(fmaf(sv[2 * i + 1], p.scale_log2, neg_m));
-        l8[(2 * i) & 7] += p0;
-        l8[(2 * i + 1) & 7] += p1;
+        float t0, t1;
+        f32x2_unpack(f32x2_fma(f32x2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), t0, t1);
+        const float p0 = ex2_approx(t0);
+        const float p1 = ex2_approx(t1);
+        l4[i & 3] = f32x2_add(l4[i & 3], f32x2_pack(p0, p1));
         pk[i] = pack_bf16x2(p0, p1);
       }
+      float l8[8];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) f32x2_unpack(l4[i], l8[2 * i], l8[2 * i + 1]);
       l_run += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
       if (j > 0) {
         if (!mbar_wait(pv_done, (j - 1) & 1, wc)) {
