@@ -51,9 +51,12 @@ def test_absorbed_weights_match_oracle():
     assert_close(f64(w_b), ref_b, what="W_B")
 
 
-@pytest.mark.parametrize("nq,batch", [(64, 1), (200, 2)])
-def test_query_prologue_matches_oracle(nq, batch):
-    w = synth.workload("tiny", batch=batch)
+@pytest.mark.parametrize("nq,batch,shape", [
+    (64, 1, {}), (200, 2, {}),
+    (130, 2, dict(d_c=128, d_r=64, rope_pairs=(12, 10, 10), rope_axis_dims=(64, 64, 64))),
+])
+def test_query_prologue_matches_oracle(nq, batch, shape):
+    w = synth.workload("tiny", batch=batch, **shape)
     wt = synth.draw_layer_weights(w, seed=72)
     dev = {k: v.cuda() for k, v in wt.items()}
     cfg = V.make_config(w)

@@ -134,6 +134,23 @@ def test_sink_window_attention_parity(case, flags):
     assert_close(f64(o), oracle_window(w, oc, q_c, q_r, q_pos), what="window o_lat")
 
 
+@pytest.mark.parametrize("d_c,d_r,pairs,dims", [(128, 64, (12, 10, 10), (64, 64, 64)),
+                                               (64, 32, (6, 5, 5), (44, 42, 42))])
+def test_sink_window_other_latent_sizes(d_c, d_r, pairs, dims):
+    """The window path at other (d_c, d_r): the assembly kernel's 16-byte
+    pieces per key and the tensor-core attention instance for that shape."""
+    w = synth.workload("tiny", grid_h=9, grid_w=10, window_frames=4, sink_frames=1, batch=2,
+                       d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims)
+    weights = synth.draw_layer_weights(w, seed=87)
+    chunks = [(f, 1) for f in range(8)]
+    cache, oc = window_chunks(w, weights, chunks)
+    T = w.tokens_per_frame
+    q_c, q_r = synth.draw_queries(w, T, 88)
+    q_pos = synth.grid_positions(w, 7, 1)
+    o = window_forward(w, cache, q_c, q_r, q_pos)
+    assert_close(f64(o), oracle_window(w, oc, q_c, q_r, q_pos), what=f"window o_lat {d_c}/{d_r}")
+
+
 def test_contiguous_window_matches_rotate_at_append_path():
     """No sink: re-indexed rotate-at-use attention equals the rotate-at-append
     hot path on the same inputs (RoPE relativity), after the ring wrapped."""
