@@ -402,7 +402,8 @@ unsigned long long mla_query_workspace_bytes(const mla_config* cfg, int Nq) {
   if (check_config(cfg) != MLA_OK || Nq < 1 || cfg->d_q <= 0) return 0;
   const unsigned long long rows = static_cast<unsigned long long>(cfg->batch) * Nq;
   const unsigned long long ct = (rows * cfg->d_q * 2 + 255) / 256 * 256;
-  return ct + static_cast<unsigned long long>((cfg->d_q + 255) / 256) * rows * 4;
+  return ct + static_cast<unsigned long long>((cfg->d_q + kQuerySqTile - 1) / kQuerySqTile) *
+                  rows * 4;
 }
 
 int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq, const void* w_qcat,

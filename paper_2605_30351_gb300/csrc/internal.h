@@ -8,6 +8,10 @@
 
 namespace vmla {
 
+// Column-tile width of the query prologue's first GEMM, which also sets how
+// many partial sums of squares per row the workspace holds (ceil(d_q / it)).
+constexpr int kQuerySqTile = 192;
+
 // First slot of latent frame f: sink frames (f < S) keep slot f*T for good,
 // later frames share the W - S remaining frame slots in FIFO order
 // (App. D.4). With S = 0 this is the ring (f mod W)*T.

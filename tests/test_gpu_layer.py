@@ -139,3 +139,29 @@ def test_output_projection_at_wan_size(batch):
     flat = f64(o_lat).reshape(batch, w.chunk_tokens, -1)[:, rows]
     ref = flat @ f64(w_b).T
     assert_close(f64(y)[:, rows], ref, what=f"y, batch {batch}")
+
+
+@pytest.mark.parametrize("batch", [1, 2])
+def test_query_prologue_at_wan_size(batch):
+    """The prologue at one and two Wan chunks (the first GEMM's two tile
+    widths), checked against the oracle on sampled tokens."""
+    w = synth.workload("wan", batch=batch)
+    wt = synth.draw_layer_weights(w, seed=97)
+    dev = {k: v.cuda() for k, v in wt.items()}
+    cfg = V.make_config(w)
+    w_qcat, _ = V.mla_absorb_weights(cfg, dev["w_uq"], dev["w_uk"], dev["w_qr"], dev["gamma_q"],
+                                     dev["w_uv"], dev["w_o"])
+    nq = w.chunk_tokens
+    x = synth.draw_tokens(w, nq, 98)
+    ws = torch.empty(V.mla_query_workspace_bytes(cfg, nq), dtype=torch.uint8, device="cuda")
+    q_c = torch.empty(batch, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    q_r = torch.empty(batch, nq, w.heads, w.d_r, dtype=torch.bfloat16, device="cuda")
+    V.mla_query_prologue(cfg, x.cuda(), dev["w_dq"], w_qcat, ws, q_c, q_r)
+    torch.cuda.synchronize()
+    tok = np.array([0, 1, 127, 128, 3000, nq - 1])
+    w64 = weights64(wt)
+    c_q = O.rmsnorm(f64(x[:, tok]) @ w64["w_dq"].T, w64["gamma_q"], w.rms_eps)
+    ref_qc = np.stack([O.absorb_query(c_q[b], w64["w_uq"], w64["w_uk"]) for b in range(batch)])
+    ref_qr = np.einsum("hrq,bnq->bnhr", w64["w_qr"], c_q)
+    assert_close(f64(q_c[:, tok]), ref_qc, what="q_c at Wan size")
+    assert_close(f64(q_r[:, tok]), ref_qr, what="q_r at Wan size")
