@@ -794,7 +794,8 @@ def run_memcap(args, rank):
         row["fits_budget"] = bool(used <= budget)
         fl_row = (4 * w.d_c + 2 * w.d_r) if layout == "mla" else 4 * w.head_dim
         fl = 1.0 * B * nq * w.heads * w.slots * fl_row
-        tc = layout == "dense" or (w.d_c, w.d_r) in ((64, 32), (128, 32), (192, 32), (256, 32))
+        tc = layout == "dense" or (w.d_c, w.d_r) in ((64, 32), (128, 32), (192, 32), (256, 32),
+                                                     (512, 32))
         if B > 0 and tc:
             if layout == "mla":
                 c0 = caches[0]

@@ -152,6 +152,10 @@ int mla_cache_reset(mla_cache* cache, void* stream);
  * the range reaches the newest frame: extend the window or rewrite the
  * current chunk, as each denoising step does). Afterwards
  * frames_written = first_frame + n_frames.
+ * Tensor-core kernel for d_c in {64, 128, 192, 256, 512} and d_r in {32, 64}
+ * with hidden a multiple of 64 (at d_c = 512 the c and k^R halves run in
+ * separate CTAs); other shapes return MLA_ERR_UNSUPPORTED unless
+ * MLA_FLAG_SIMT selects the SIMT kernel.
  */
 int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv,
                      const void* gamma_kv, const void* w_kr, const int* pos,
@@ -172,6 +176,9 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv,
  * chunk, so the chunk-causal mask (App. D.4) keeps every valid slot.
  * MLA_ERR_ARG if no slot is valid, Nq < 1, or the cache keeps k^R unrotated
  * (MLA_FLAG_ROTATE_AT_USE: use mla_attention_window_forward).
+ * Tensor-core kernel for d_c in {64, 128, 192, 256, 512} and d_r in {32, 64}
+ * (at d_c = 512 two CTAs share each 128-row tile, 256 output columns each);
+ * other shapes return MLA_ERR_UNSUPPORTED unless MLA_FLAG_SIMT is set.
  */
 int mla_attention_forward(const mla_cache* cache, const void* q_c,
                           const void* q_r, const int* q_pos, int Nq,

@@ -12,6 +12,10 @@
 //              cache keeps k^R unrotated), bf16, 16-byte stores into the
 //              token's slot: (f mod W) * T + k, or with S sink frames f * T + k
 //              for f < S and (S + (f - S) mod (W - S)) * T + k after them.
+// For d_c = 512 the [128 x (d_c + d_r)] accumulator does not fit the 512
+// TMEM columns; the launch then runs two CTAs per token tile (blockIdx.z):
+// one accumulates c (two N = 256 MMAs per K step) and applies RMSNorm, the
+// other accumulates k^R and applies RoPE. Both stream the same x tile.
 #include <cmath>
 
 #include "internal.h"
@@ -24,10 +28,18 @@ constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kThreads = 192;
 
-template <int DC, int DR>
+// What one CTA computes: both parts (d_c <= 256), or, for d_c = 512 whose
+// [d_c + d_r] accumulator exceeds TMEM, only c or only k^R (the two CTAs of
+// a token tile need nothing from each other: RMSNorm runs over c alone).
+enum AppendPart { kPartBoth = 0, kPartC = 1, kPartK = 2 };
+
+template <int DC, int DR, int PART = kPartBoth>
 struct AppendShape {
-  static constexpr int N = DC + DR;
-  static constexpr bool kSplitN = N > 256;  // then two MMAs: c part and k part
+  static constexpr int NC = PART == kPartK ? 0 : DC;  // c columns of the accumulator
+  static constexpr int NK = PART == kPartC ? 0 : DR;  // k^R columns, after c
+  static constexpr int N = NC + NK;
+  static constexpr bool kSplitN = N > 256;  // then MMAs of at most 256: c part(s), k part
+  static constexpr int kWcBox = DC < 256 ? DC : 256;  // W_dkv rows per TMA box
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = N * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
@@ -35,11 +47,13 @@ struct AppendShape {
   static constexpr int kFit = (232448 - 1024 - kBarBytes) / kStageBytes;
   static constexpr int kStages = kFit > 6 ? 6 : kFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
-  static constexpr uint32_t kTmemCols = N <= 256 ? 256 : 512;
+  static constexpr uint32_t kTmemCols = N <= 32 ? 32 : (N <= 64 ? 64 : (N <= 256 ? 256 : 512));
   // output staging row: N bf16 plus 16 bytes, so rows start on different banks
   static constexpr int kOutStride = N * 2 + 16;
   static_assert(kBM * kOutStride + kBM * 8 <= kStages * kStageBytes, "staging fits in the ring");
-  static_assert(DC % 32 == 0 && DR % 32 == 0 && DC <= 256 && DR <= 64, "shape");
+  static_assert(DC % 32 == 0 && DR % 32 == 0 && DR <= 64 && (DC <= 256 || DC % 256 == 0),
+                "shape");
+  static_assert(PART == kPartBoth || DC > 256, "parts are split only when d_c > 256");
   static_assert(N <= 512, "accumulator must fit in TMEM");
   static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
   static_assert(kStages >= 2, "smem");
@@ -58,12 +72,12 @@ struct AppendKParams {
   int* status;
 };
 
-template <int DC, int DR>
-__global__ void __launch_bounds__(kThreads, 1)
-    mla_append_tc_kernel(const __grid_constant__ CUtensorMap tm_x,
-                         const __grid_constant__ CUtensorMap tm_wc,
-                         const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
-  using S = AppendShape<DC, DR>;
+template <int DC, int DR, int PART>
+__device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUtensorMap* tm_wc,
+                                            const CUtensorMap* tm_wk, const AppendKParams& p) {
+  using S = AppendShape<DC, DR, PART>;
+  constexpr int NC = S::NC;
+  constexpr int NK = S::NK;
   constexpr int NST = S::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_smem_1024(smem_raw);
@@ -100,9 +114,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      tma_prefetch_desc(&tm_x);
-      tma_prefetch_desc(&tm_wc);
-      tma_prefetch_desc(&tm_wk);
+      tma_prefetch_desc(tm_x);
+      if constexpr (NC > 0) tma_prefetch_desc(tm_wc);
+      if constexpr (NK > 0) tma_prefetch_desc(tm_wk);
       int issued = 0;
       for (int kb = 0; kb < p.k_blocks; ++kb) {
         const int st = kb % NST;
@@ -110,9 +124,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint8_t* a = smem + st * S::kStageBytes;
         uint8_t* bm = a + S::kABytes;
         mbar_arrive_expect_tx(&full[st], S::kStageBytes);
-        tma_load_3d(a, &tm_x, &full[st], kb * kBK, row0, b);
-        tma_load_2d(bm, &tm_wc, &full[st], kb * kBK, 0);
-        tma_load_2d(bm + DC * 128, &tm_wk, &full[st], kb * kBK, 0);
+        tma_load_3d(a, tm_x, &full[st], kb * kBK, row0, b);
+        if constexpr (NC > 0)
+          for (int h = 0; h < NC / S::kWcBox; ++h)
+            tma_load_2d(bm + h * S::kWcBox * 128, tm_wc, &full[st], kb * kBK, h * S::kWcBox);
+        if constexpr (NK > 0) tma_load_2d(bm + NC * 128, tm_wk, &full[st], kb * kBK, 0);
         issued = kb + 1;
       }
       if (*abort_flag)
@@ -139,10 +155,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             constexpr uint32_t idesc = idesc_bf16_f32(kBM, S::N, false, false);
             umma_ss(tmem, ad, sdesc(ba + k * 32, 16, 1024, kSw128), idesc, acc);
           } else {
-            constexpr uint32_t idesc_c = idesc_bf16_f32(kBM, DC, false, false);
-            constexpr uint32_t idesc_k = idesc_bf16_f32(kBM, DR, false, false);
-            umma_ss(tmem, ad, sdesc(ba + k * 32, 16, 1024, kSw128), idesc_c, acc);
-            umma_ss(tmem + DC, ad, sdesc(ba + DC * 128 + k * 32, 16, 1024, kSw128), idesc_k, acc);
+            constexpr int kHc = NC < 256 ? NC : 256;  // columns per c MMA
+            constexpr uint32_t idesc_c = idesc_bf16_f32(kBM, kHc, false, false);
+#pragma unroll
+            for (int h = 0; h < NC / kHc; ++h)
+              umma_ss(tmem + h * kHc, ad, sdesc(ba + h * kHc * 128 + k * 32, 16, 1024, kSw128),
+                      idesc_c, acc);
+            if constexpr (NK > 0) {
+              constexpr uint32_t idesc_k = idesc_bf16_f32(kBM, NK, false, false);
+              umma_ss(tmem + NC, ad, sdesc(ba + NC * 128 + k * 32, 16, 1024, kSw128), idesc_k,
+                      acc);
+            }
           }
         }
         umma_commit(&empty[st]);
@@ -169,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // pass 1: mean square of c over d_c (fp32)
       float ss = 0.f;
 #pragma unroll 1
-      for (int cb = 0; cb < DC / 32; ++cb) {
+      for (int cb = 0; cb < NC / 32; ++cb) {
         uint32_t v[32];
         tmem_ld32(t_row + cb * 32, v);
         tmem_wait_ld();
@@ -186,7 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint8_t* srow = stage_out + r * S::kOutStride;
       // pass 2: gamma * c / rms -> bf16
 #pragma unroll 1
-      for (int cb = 0; cb < DC / 32; ++cb) {
+      for (int cb = 0; cb < NC / 32; ++cb) {
         uint32_t v[32];
         tmem_ld32(t_row + cb * 32, v);
         tmem_wait_ld();
@@ -209,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // positional key: RoPE3D at the token's (t, h, w), or unrotated
       int pa[3] = {0, 0, 0};
-      if (row_ok && p.rotate) {
+      if (NK > 0 && row_ok && p.rotate) {
         const int* pp = p.pos + (static_cast<size_t>(b) * p.n_tok + n) * 3;
         pa[0] = __ldg(pp);
         pa[1] = __ldg(pp + 1);
@@ -222,9 +245,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
       }
 #pragma unroll 1
-      for (int cb = 0; cb < DR / 32; ++cb) {
+      for (int cb = 0; cb < NK / 32; ++cb) {
         uint32_t v[32];
-        tmem_ld32(t_row + DC + cb * 32, v);
+        tmem_ld32(t_row + NC + cb * 32, v);
         tmem_wait_ld();
         uint32_t pk[16];
 #pragma unroll
@@ -238,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-          *reinterpret_cast<uint4*>(srow + DC * 2 + cb * 64 + i * 16) =
+          *reinterpret_cast<uint4*>(srow + NC * 2 + cb * 64 + i * 16) =
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
     }
@@ -246,7 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("bar.sync 1, 128;" ::: "memory");
     if (have_acc) {
       constexpr int kChunks = S::N * 2 / 16;  // 16-byte pieces per output row
-      constexpr int kChunksC = DC * 2 / 16;
+      constexpr int kChunksC = NC * 2 / 16;
       for (int q = r; q < kBM * kChunks; q += kBM) {
         const int row = q / kChunks, ch = q % kChunks;
         const long long slot = slot_of[row];
@@ -270,18 +293,46 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int DC, int DR>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_append_tc_kernel(const __grid_constant__ CUtensorMap tm_x,
+                         const __grid_constant__ CUtensorMap tm_wc,
+                         const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
+  append_body<DC, DR, kPartBoth>(&tm_x, &tm_wc, &tm_wk, p);
+}
+
+// d_c > 256: blockIdx.z = 0 computes c, 1 computes k^R, for the same tokens
+template <int DC, int DR>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_append_tc_split_kernel(const __grid_constant__ CUtensorMap tm_x,
+                               const __grid_constant__ CUtensorMap tm_wc,
+                               const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
+  if (blockIdx.z == 0)
+    append_body<DC, DR, kPartC>(&tm_x, &tm_wc, &tm_wk, p);
+  else
+    append_body<DC, DR, kPartK>(&tm_x, &tm_wc, &tm_wk, p);
+}
+
+template <int DC, int DR>
 int launch_tc(const AppendArgs& a) {
-  using S = AppendShape<DC, DR>;
+  constexpr bool kSplit = DC > 256;
+  using S = AppendShape<DC, DR, kSplit ? kPartC : kPartBoth>;
+  using SK = AppendShape<DC, DR, kSplit ? kPartK : kPartBoth>;
+  constexpr int kSmem = S::kSmemBytes > SK::kSmemBytes ? S::kSmemBytes : SK::kSmemBytes;
   CUtensorMap tm_x, tm_wc, tm_wk;
   const unsigned long long H = a.hidden, n_tok = a.n_tok;
   if (!encode_map_3d_bf16(&tm_x, a.x, H, n_tok, a.batch, H * 2, n_tok * H * 2, kBK, kBM,
                           CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !encode_map_2d_bf16(&tm_wc, a.w_dkv, H, DC, H * 2, kBK, DC, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_2d_bf16(&tm_wc, a.w_dkv, H, DC, H * 2, kBK, S::kWcBox,
+                          CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_wk, a.w_kr, H, DR, H * 2, kBK, DR, CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
-  auto kern = mla_append_tc_kernel<DC, DR>;
-  cudaError_t e =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
+  auto kern = [] {
+    if constexpr (kSplit)
+      return mla_append_tc_split_kernel<DC, DR>;
+    else
+      return mla_append_tc_kernel<DC, DR>;
+  }();
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return MLA_ERR_CUDA;
@@ -306,8 +357,8 @@ int launch_tc(const AppendArgs& a) {
   kp.use_rmsnorm = a.use_rmsnorm;
   kp.eps = a.eps;
   kp.status = a.status;
-  const dim3 grid((a.n_tok + kBM - 1) / kBM, a.batch);
-  kern<<<grid, kThreads, S::kSmemBytes, a.stream>>>(tm_x, tm_wc, tm_wk, kp);
+  const dim3 grid((a.n_tok + kBM - 1) / kBM, a.batch, kSplit ? 2 : 1);
+  kern<<<grid, kThreads, kSmem, a.stream>>>(tm_x, tm_wc, tm_wk, kp);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
@@ -326,6 +377,7 @@ int launch_append_tc(const AppendArgs& a) {
       case 128: return launch_tc<128, 32>(a);
       case 192: return launch_tc<192, 32>(a);
       case 256: return launch_tc<256, 32>(a);
+      case 512: return launch_tc<512, 32>(a);
       default: break;
     }
   } else if (a.d_r == 64) {
@@ -334,6 +386,7 @@ int launch_append_tc(const AppendArgs& a) {
       case 128: return launch_tc<128, 64>(a);
       case 192: return launch_tc<192, 64>(a);
       case 256: return launch_tc<256, 64>(a);
+      case 512: return launch_tc<512, 64>(a);
       default: break;
     }
   }

@@ -34,6 +34,13 @@
 // When Q does not fit there (d_c = 256 with BN = 128) it stays in shared memory
 // (TMA-loaded q_c plus the rotated q_r stored by the softmax warps) and QK
 // reads it there.
+// d_c = 512: a 512-column fp32 O alone fills TMEM, so each 128-row tile runs
+// on a cluster of two CTAs, each owning 256 output columns (DV). Both score
+// the full [c | k] tile (QK is computed twice, PV once: 2112 useful of 3200
+// issued FLOP per row-key pair) and share every key tile through the same
+// multicast as the row-tile pairs above; each keeps the q_c columns that fit
+// next to S, P and its O half in TMEM (320) and the rest of Q in shared
+// memory, so QK mixes TMEM- and shared-memory A operands.
 // The V operand is the first d_c columns of the same key tile read MN-major,
 // so the cache is never expanded into per-head keys or values.
 #include <cmath>
@@ -48,19 +55,27 @@ constexpr int kBM = 128;       // rows per CTA = TMEM lanes
 constexpr int kThreads = 224;  // 7 warps
 constexpr float kRescaleLog2 = 8.0f;
 
-template <int DC, int DR, int BN>
+template <int DC, int DR, int BN, int DV = DC>
 struct AttnShape {
   static constexpr int kBN = BN;                   // keys per block
   static constexpr int DK = DC + DR;
-  static constexpr int kTileBytes = kBN * DK * 2;  // one key stage (and the smem Q tile)
+  static constexpr int kSplit = DC / DV;           // CTAs per row tile, DV output columns each
+  static constexpr int kTileBytes = kBN * DK * 2;  // one key stage
   static constexpr int kCBox = kBN * 128;          // one [BN keys x 64 columns] box of c
   static constexpr int kKrOff = DC * kBN * 2;      // byte offset of the d_r columns in a tile
   static constexpr int kTmemS = 0;
   static constexpr int kTmemP = kBN;               // bf16 P: two values per column
   static constexpr int kTmemO = kBN + kBN / 2;
-  static constexpr int kTmemQ = kTmemO + DC;
+  static constexpr int kTmemQ = kTmemO + DV;
   static constexpr bool kQinTmem = kTmemQ + DK / 2 <= 512;
-  static constexpr int kQBytes = kQinTmem ? 0 : kBM * DK * 2;
+  // q_c columns held in TMEM: all of them when Q fits; with a split output
+  // the leading 64-column boxes that fit, the rest of Q in shared memory
+  static constexpr int kQcTmem =
+      kQinTmem ? DC : (kSplit > 1 ? ((512 - kTmemQ) * 2 / 64) * 64 : 0);
+  static constexpr int kQcSmem = DC - kQcTmem;
+  // shared-memory Q tile: [128 rows x 64 columns] boxes of q_c, then q_r
+  static constexpr int kQKrOff = kQcSmem * kBM * 2;
+  static constexpr int kQBytes = kQinTmem ? 0 : kQKrOff + kBM * DR * 2;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmemCap = 232448;
   static constexpr int kFit = (kSmemCap - 1024 - kBarBytes - kQBytes) / kTileBytes;
@@ -72,14 +87,17 @@ struct AttnShape {
   static constexpr uint32_t kKrRow = DR * 2;      // bytes per row of the d_r block
   static constexpr uint32_t kKrSbo = 8 * kKrRow;  // one 8-row swizzle atom
   static constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
-  static constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, DC, false, true);
-  static_assert(kQinTmem || kBM == kBN, "the smem Q tile and a key stage share one layout");
+  static constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, DV, false, true);
   static_assert(BN == 128 || BN == 64, "key block: 128 or 64");
-  static_assert(DC % 64 == 0 && DC >= 64 && DC <= 256, "d_c: multiple of 64 up to 256");
+  static_assert(DC % 64 == 0 && DC >= 64 && DV % 64 == 0 && DV <= 256 && DC % DV == 0,
+                "d_c: multiple of 64; each CTA's output columns: multiple of 64 up to 256");
+  static_assert(kSplit == 1 || kSplit == 2, "output split over at most two CTAs");
   static_assert(DR == 32 || DR == 64, "d_r: 32 or 64");
-  static_assert(kTmemO + DC <= 512, "S, P and O must fit in 512 TMEM columns");
+  static_assert(kTmemO + DV <= 512 && kTmemQ + kQcTmem / 2 <= 512,
+                "S, P, O and the TMEM part of Q must fit in 512 TMEM columns");
   static_assert(kStages >= 2, "at least two key stages must fit in shared memory");
-  static_assert(kTileBytes % 1024 == 0 && kKrOff % 1024 == 0, "swizzle-atom alignment");
+  static_assert(kTileBytes % 1024 == 0 && kKrOff % 1024 == 0 && kQKrOff % 1024 == 0,
+                "swizzle-atom alignment");
 };
 
 struct AttnKParams {
@@ -93,16 +111,18 @@ struct AttnKParams {
   int* status;
 };
 
-template <int DC, int DR, int CL, int BN>
+template <int DC, int DR, int CL, int BN, int DV>
 __global__ void __launch_bounds__(kThreads, 1)
     mla_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_qc,
                        const __grid_constant__ CUtensorMap tm_c,
                        const __grid_constant__ CUtensorMap tm_kr, const AttnKParams p) {
-  using S = AttnShape<DC, DR, BN>;
+  using S = AttnShape<DC, DR, BN, DV>;
   constexpr int kBN = S::kBN;
   constexpr int NST = S::kStages;
   constexpr uint16_t kPair = static_cast<uint16_t>((1u << CL) - 1u);  // every CTA of the cluster
   static_assert(CL == 1 || CL == 2, "clusters of one or two CTAs");
+  // a split row tile's CTAs form the cluster: both read every key tile
+  static_assert(S::kSplit == 1 || CL == S::kSplit, "split CTAs share one cluster");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_smem_1024(smem_raw);
   uint8_t* sQ = smem;  // only when Q stays in shared memory
@@ -123,7 +143,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.y;
-  const int row0 = blockIdx.x * kBM;
+  const int tile = blockIdx.x / S::kSplit;
+  const int vpart = blockIdx.x - tile * S::kSplit;  // which DV output columns
+  const int row0 = tile * kBM;
   const int nblk = (p.n_valid + kBN - 1) / kBN;
   const WaitCtx wc{abort_flag, p.status};
 
@@ -162,9 +184,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_kr);
       if constexpr (!S::kQinTmem) {
         tma_prefetch_desc(&tm_qc);
-        mbar_arrive_expect_tx(q_tma_full, DC * kBM * 2);
-        for (int cb = 0; cb < DC / 64; ++cb)
-          tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, cb * 64, row0, b);
+        mbar_arrive_expect_tx(q_tma_full, S::kQcSmem * kBM * 2);
+        for (int cb = 0; cb < S::kQcSmem / 64; ++cb)
+          tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, S::kQcTmem + cb * 64, row0, b);
       }
       int issued = 0;
       for (int j = 0; j < nblk; ++j) {
@@ -223,10 +245,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < 4; ++k) {
             const uint64_t bd = sdesc(ka + cb * S::kCBox + k * 32, 16, 1024, kSw128);
             const uint32_t acc = (cb | k) != 0 ? 1u : 0u;
-            if constexpr (S::kQinTmem)
+            if (cb < S::kQcTmem / 64)  // resolved at compile time (unrolled)
               umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + (cb * 4 + k) * 8, bd, S::kIdescQK, acc);
             else
-              umma_ss(tmem + S::kTmemS, sdesc(qa + cb * 16384 + k * 32, 16, 1024, kSw128), bd,
+              umma_ss(tmem + S::kTmemS,
+                      sdesc(qa + (cb - S::kQcTmem / 64) * 16384 + k * 32, 16, 1024, kSw128), bd,
                       S::kIdescQK, acc);
           }
 #pragma unroll
@@ -235,8 +258,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           if constexpr (S::kQinTmem)
             umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + DC / 2 + k * 8, bd, S::kIdescQK, 1u);
           else
-            umma_ss(tmem + S::kTmemS, sdesc(qa + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw), bd,
-                    S::kIdescQK, 1u);
+            umma_ss(tmem + S::kTmemS, sdesc(qa + S::kQKrOff + k * 32, 16, S::kKrSbo, S::kKrSw),
+                    bd, S::kIdescQK, 1u);
         }
         umma_commit(s_full);
       }
@@ -251,14 +274,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       bool ok = true;
       for (int i = 0; ok && i < nblk; ++i) {
-        // O += P_i V_i, V = the first d_c columns of block i's stage (MN-major)
+        // O += P_i V_i, V = this CTA's DV of the first d_c columns of block
+        // i's stage (MN-major)
         if (!mbar_wait(p_full, i & 1, wc)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const int st = i % NST;
-        const uint32_t va = smem_u32(sKV) + st * S::kTileBytes;
+        const uint32_t va = smem_u32(sKV) + st * S::kTileBytes + vpart * (DV / 64) * S::kCBox;
 #pragma unroll
         for (int s = 0; s < kBN / 16; ++s)
           umma_ts(tmem + S::kTmemO, tmem + S::kTmemP + s * 8,
@@ -317,12 +341,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           w[i] = pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x);
         }
       }
-      if constexpr (S::kQinTmem) {
+      if constexpr (S::kQcTmem > 0) {
         // TMEM holds the MMA's A operand row-major: column c = elements 2c, 2c+1
         const uint4* qsrc = reinterpret_cast<const uint4*>(
             p.q_c + (static_cast<size_t>(b) * p.rows + (row_ok ? grow : 0)) * DC);
 #pragma unroll
-        for (int c = 0; c < DC / 64; ++c) {
+        for (int c = 0; c < S::kQcTmem / 64; ++c) {
           uint32_t qw[32];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
@@ -334,14 +358,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tmem_st32(tmem + t_lane + S::kTmemQ + c * 32, qw);
         }
+      }
+      if constexpr (S::kQinTmem) {
 #pragma unroll
         for (int c = 0; c < DR / 32; ++c)
           tmem_st16(tmem + t_lane + S::kTmemQ + DC / 2 + c * 16, w + c * 16);
-        tmem_wait_st();
-        tc_fence_before();
       } else {
         // the same 16-byte-chunk swizzle the TMA applies to the q_c part
-        uint8_t* krow = sQ + S::kKrOff + r * S::kKrRow;
+        uint8_t* krow = sQ + S::kQKrOff + r * S::kKrRow;
 #pragma unroll
         for (int c = 0; c < DR / 8; ++c) {
           const int phys = DR == 32 ? (c ^ ((r >> 1) & 3)) : (c ^ (r & 7));
@@ -349,6 +373,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
         }
         fence_proxy_async_smem();
+      }
+      if constexpr (S::kQcTmem > 0) {
+        tmem_wait_st();
+        tc_fence_before();
       }
       mbar_arrive(q_ready);
     }
@@ -441,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         if (__any_sync(0xffffffffu, need)) {
 #pragma unroll 1
-          for (int c = 0; c < DC / 32; ++c) {
+          for (int c = 0; c < DV / 32; ++c) {
             uint32_t ov[32];
             tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
             tmem_wait_ld();
@@ -464,9 +492,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ok && mbar_wait(pv_done, (nblk - 1) & 1, wc)) {
       tc_fence_after();
       const float inv_l = 1.f / l_run;
-      uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC);
+      uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC +
+                                            vpart * DV);
 #pragma unroll 1
-      for (int c = 0; c < DC / 32; ++c) {
+      for (int c = 0; c < DV / 32; ++c) {
         uint32_t ov[32];
         tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
         tmem_wait_ld();
@@ -494,9 +523,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   if constexpr (CL > 1) cluster_sync();
 }
 
-template <int DC, int DR, int CL, int BN>
+template <int DC, int DR, int CL, int BN, int DV = DC>
 int launch_tc(const AttnArgs& a) {
-  using S = AttnShape<DC, DR, BN>;
+  using S = AttnShape<DC, DR, BN, DV>;
   CUtensorMap tm_qc, tm_c, tm_kr;
   const unsigned long long rows = a.rows, slots = a.slots;
   if (!encode_map_3d_bf16(&tm_qc, a.q_c, DC, rows, a.batch, DC * 2ull, rows * DC * 2ull, 64,
@@ -507,7 +536,7 @@ int launch_tc(const AttnArgs& a) {
                           S::kBN,
                           DR == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
-  auto kern = mla_attn_tc_kernel<DC, DR, CL, BN>;
+  auto kern = mla_attn_tc_kernel<DC, DR, CL, BN, DV>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
   if (e != cudaSuccess) {
@@ -530,7 +559,8 @@ int launch_tc(const AttnArgs& a) {
   kp.status = a.status;
   const int tiles = (a.rows + kBM - 1) / kBM;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((tiles + CL - 1) / CL * CL, a.batch, 1);  // pairs stay within a batch row
+  // pairs stay within a batch row; a split tile's CTAs are adjacent
+  cfg.gridDim = dim3((tiles * S::kSplit + CL - 1) / CL * CL, a.batch, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = S::kSmemBytes;
   cfg.stream = a.stream;
@@ -566,6 +596,7 @@ int launch_attention_tc(const AttnArgs& a) {
       case 128: return launch_tc_pick<128, 32>(a);
       case 192: return launch_tc_pick<192, 32>(a);
       case 256: return launch_tc_pick<256, 32>(a);  // Q in shared memory (faster than 64-key blocks)
+      case 512: return launch_tc<512, 32, 2, 64, 256>(a);  // output split over a CTA pair
       default: break;
     }
   } else if (a.d_r == 64) {
@@ -574,6 +605,7 @@ int launch_attention_tc(const AttnArgs& a) {
       case 128: return launch_tc_pick<128, 64>(a);
       case 192: return launch_tc_pick<192, 64>(a);
       case 256: return launch_tc_pick<256, 64, 64>(a);  // Q in TMEM needs 64-key blocks
+      case 512: return launch_tc<512, 64, 2, 64, 256>(a);
       default: break;
     }
   }

@@ -200,6 +200,89 @@ def test_attention_dc512_simt():
     assert_close(f64(o), oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid()), what="d_c=512")
 
 
+# d_c = 512: the attention output is split over a CTA pair (256 columns
+# each) and the append runs its c and k^R halves in separate CTAs
+DC512 = [(32, (6, 5, 5), (44, 42, 42)), (64, (12, 10, 10), (64, 64, 64))]
+
+
+@pytest.mark.parametrize("d_r,pairs,dims", DC512)
+def test_append_dc512_parity(d_r, pairs, dims):
+    """T = 100 (ragged tiles), batch 2, ring wrapped, RMSNorm over 512 columns."""
+    w = small(d_c=512, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims, grid_h=10, grid_w=10,
+              window_frames=4, batch=2)
+    weights = synth.draw_layer_weights(w, seed=17)
+    cache, oc = run_chunks(w, weights, [(0, 2), (2, 2), (4, 1)])
+    valid = oc.valid_slots()
+    assert len(valid) == 4 * 100
+    assert_close(f64(cache.c)[:, valid], oc.c[:, valid], what="c d_c=512")
+    assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what="k_rope d_c=512")
+
+
+def test_append_dc512_bit_exact():
+    """One-hot projections, no RMSNorm, positions zero: both halves of the
+    split append copy input values, so slots match bit for bit."""
+    w = small(d_c=512, d_r=32, rope_pairs=(6, 5, 5), grid_h=9, grid_w=9, window_frames=3,
+              batch=2)
+    cfg = V.make_config(w, V.MLA_FLAG_NO_RMSNORM)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    d, dc, dr = w.hidden, w.d_c, w.d_r
+    w_dkv = torch.zeros(dc, d, dtype=torch.bfloat16)
+    w_dkv[torch.arange(dc), torch.arange(dc)] = 1
+    w_kr = torch.zeros(dr, d, dtype=torch.bfloat16)
+    w_kr[torch.arange(dr), dc + torch.arange(dr)] = 1
+    T = w.tokens_per_frame
+    frames = {}
+    for i, (first, n) in enumerate([(0, 2), (2, 2), (4, 1)]):
+        x = synth.draw_tokens(w, n * T, 520 + i)
+        pos = torch.zeros(w.batch, n * T, 3, dtype=torch.int32)
+        V.mla_cache_append(cache, x.cuda(), w_dkv.cuda(), None, w_kr.cuda(), pos.cuda(), first, n)
+        for k in range(n):
+            frames[first + k] = x[:, k * T:(k + 1) * T]
+    torch.cuda.synchronize()
+    c_bits = cache.c.cpu().view(torch.int16)
+    k_bits = cache.kr.cpu().view(torch.int16)
+    for f in O.window_frames(cache.frames_written, w.window_frames):
+        s0 = O.ring_slot(f, 0, T, w.window_frames)
+        xb = frames[f].view(torch.int16)
+        assert torch.equal(c_bits[:, s0:s0 + T], xb[:, :, :dc]), f
+        assert torch.equal(k_bits[:, s0:s0 + T], xb[:, :, dc:dc + dr]), f
+
+
+@pytest.mark.parametrize("d_r,pairs,dims", DC512)
+def test_attention_dc512_parity(d_r, pairs, dims):
+    """390 keys (six 64-key blocks and a ragged one), 480 rows (a ragged
+    fourth row tile), batch 2."""
+    w = small(d_c=512, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims, grid_h=10, grid_w=13,
+              window_frames=3, batch=2)
+    cache, c, k = upload_cache(w, 15, 3)
+    q_c, q_r = synth.draw_queries(w, 40, 16)
+    q_pos = synth.grid_positions(w, 2, 1)[:, :40].contiguous()
+    o = torch.empty(w.batch, 40, w.heads, 512, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    assert_close(f64(o), oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid()),
+                 what=f"d_c=512 d_r={d_r}")
+
+
+def test_attention_dc512_wan_sampled_rows():
+    """Wan shape with d_c = 512 (4680 x 12 rows, 32760 keys), sampled rows,
+    including both output halves of the first and last row tiles."""
+    w = synth.workload("wan").with_(d_c=512)
+    cache, c, k = upload_cache(w, 35, w.window_frames)
+    q_c, q_r = synth.draw_queries(w, w.chunk_tokens, 36)
+    q_pos = synth.grid_positions(w, 18, 3)
+    o = torch.empty(1, w.chunk_tokens, w.heads, 512, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(1)
+    rows = np.sort(rng.choice(w.chunk_tokens * w.heads, 48, replace=False))
+    rows = np.concatenate([[0, 127], rows, [w.chunk_tokens * w.heads - 1]])
+    ref = oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid(), rows=rows)
+    got = f64(o).reshape(1, -1, 512)[:, rows]
+    assert_close(got, ref, what="d_c=512 Wan rows")
+
+
 def test_tc_matches_simt_wan_rows():
     """Tensor-core and SIMT kernels agree at the full Wan-1.3B layer shape."""
     w = synth.workload("wan")
