@@ -8,9 +8,7 @@
 //     P   = exp2(S * log2(e)/sqrt(d_h) - m)        online, fp32
 //     O  += P . c                                  N = d_c (192), latent output
 // One CTA owns 128 rows (one TMEM lane each) and walks the window in blocks
-// of BN keys (128; 64 for (d_c, d_r) = (256, 64), where a 128-row Q tile fits
-// neither TMEM next to 128-key S and P buffers nor shared memory next to two
-// key stages):
+// of BN keys (128; 64 for d_c = 512):
 //   warp 0     TMA producer: [c | k] tiles into a ring of shared-memory
 //              stages (c with 128-byte swizzle, k with 64-byte swizzle).
 //              CTAs run in pairs (a cluster of two consecutive row tiles of
@@ -31,9 +29,11 @@
 //              rescales O in TMEM only when its running max grows by more
 //              than 2^8, and finally writes O / l as bf16.
 // TMEM columns: S [0,BN) P [BN,3BN/2) O [3BN/2,3BN/2+d_c) Q [3BN/2+d_c, +(d_c+d_r)/2).
-// When Q does not fit there (d_c = 256 with BN = 128) it stays in shared memory
-// (TMA-loaded q_c plus the rotated q_r stored by the softmax warps) and QK
-// reads it there.
+// When Q does not fit there (d_c = 256) it stays in shared memory (TMA-loaded
+// q_c plus the rotated q_r stored by the softmax warps) and QK reads it there;
+// where that leaves room for fewer than two key stages ((256, 64)), the first
+// q_c columns go to the TMEM left after O and QK mixes TMEM and shared-memory
+// A operands.
 // d_c = 512: a 512-column fp32 O alone fills TMEM, so each 128-row tile runs
 // on a cluster of two CTAs, each owning 256 output columns (DV). Both score
 // the full [c | k] tile (QK is computed twice, PV once: 2112 useful of 3200
@@ -67,17 +67,20 @@ struct AttnShape {
   static constexpr int kTmemP = kBN;               // bf16 P: two values per column
   static constexpr int kTmemO = kBN + kBN / 2;
   static constexpr int kTmemQ = kTmemO + DV;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kSmemCap = 232448;
   static constexpr bool kQinTmem = kTmemQ + DK / 2 <= 512;
-  // q_c columns held in TMEM: all of them when Q fits; with a split output
-  // the leading 64-column boxes that fit, the rest of Q in shared memory
+  // Where Q lives when it does not fit in TMEM: all of it in shared memory
+  // if two key stages still fit beside it (SS score MMAs measured faster
+  // than a TS/SS mix there), else the leading 64-column boxes of q_c that
+  // fit go to TMEM and the rest of Q to shared memory
+  static constexpr bool kQSmemFits = 1024 + kBarBytes + kBM * DK * 2 + 2 * kTileBytes <= kSmemCap;
   static constexpr int kQcTmem =
-      kQinTmem ? DC : (kSplit > 1 ? ((512 - kTmemQ) * 2 / 64) * 64 : 0);
+      kQinTmem ? DC : (kQSmemFits ? 0 : ((512 - kTmemQ) * 2 / 64) * 64);
   static constexpr int kQcSmem = DC - kQcTmem;
   // shared-memory Q tile: [128 rows x 64 columns] boxes of q_c, then q_r
   static constexpr int kQKrOff = kQcSmem * kBM * 2;
   static constexpr int kQBytes = kQinTmem ? 0 : kQKrOff + kBM * DR * 2;
-  static constexpr int kBarBytes = 256;
-  static constexpr int kSmemCap = 232448;
   static constexpr int kFit = (kSmemCap - 1024 - kBarBytes - kQBytes) / kTileBytes;
   static constexpr int kMaxStages = BN == 128 ? 4 : 6;
   static constexpr int kStages = kFit > kMaxStages ? kMaxStages : kFit;
@@ -604,7 +607,7 @@ int launch_attention_tc(const AttnArgs& a) {
       case 64: return launch_tc_pick<64, 64>(a);
       case 128: return launch_tc_pick<128, 64>(a);
       case 192: return launch_tc_pick<192, 64>(a);
-      case 256: return launch_tc_pick<256, 64, 64>(a);  // Q in TMEM needs 64-key blocks
+      case 256: return launch_tc_pick<256, 64>(a);  // Q split between TMEM and shared memory
       case 512: return launch_tc<512, 64, 2, 64, 256>(a);
       default: break;
     }
