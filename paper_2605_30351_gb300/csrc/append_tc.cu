@@ -17,6 +17,7 @@
 // one accumulates c (two N = 256 MMAs per K step) and applies RMSNorm, the
 // other accumulates k^R and applies RoPE. Both stream the same x tile.
 #include <cmath>
+#include <type_traits>
 
 #include "internal.h"
 #include "ptx_sm103.cuh"
@@ -28,34 +29,53 @@ constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kThreads = 192;
 
-// What one CTA computes: both parts (d_c <= 256), or, for d_c = 512 whose
-// [d_c + d_r] accumulator exceeds TMEM, only c or only k^R (the two CTAs of
-// a token tile need nothing from each other: RMSNorm runs over c alone).
-enum AppendPart { kPartBoth = 0, kPartC = 1, kPartK = 2 };
-
-template <int DC, int DR, int PART = kPartBoth>
+// What one CTA computes: NC columns of c, from column c0 (given at run time),
+// and NK columns of k^R, into one [128 x (NC + NK)] TMEM accumulator:
+//  - both parts, NC = d_c and NK = d_r (d_c <= 256);
+//  - d_c = 512, whose [d_c + d_r] accumulator exceeds TMEM: c alone or k^R
+//    alone, two CTAs per token tile that need nothing from each other
+//    (RMSNorm runs over c alone);
+//  - a grid too small to occupy the SMs (one chunk at batch 1): a cluster
+//    of CL = d_c/64 CTAs per token tile, one per 64 columns of c, the last
+//    also computing k^R, so that each SM streams the token tile and only its
+//    share of the weights. The CTAs share each x box through TMA multicast
+//    (each fetches a part of it from L2 for all) and exchange their partial
+//    RMSNorm sums of squares through distributed shared memory.
+template <int DC, int DR, int NC, int NK, int CL = 1>
 struct AppendShape {
-  static constexpr int NC = PART == kPartK ? 0 : DC;  // c columns of the accumulator
-  static constexpr int NK = PART == kPartC ? 0 : DR;  // k^R columns, after c
   static constexpr int N = NC + NK;
   static constexpr bool kSplitN = N > 256;  // then MMAs of at most 256: c part(s), k part
-  static constexpr int kWcBox = DC < 256 ? DC : 256;  // W_dkv rows per TMA box
+  static constexpr int kWcBox = NC == 0 ? 64 : (NC < 256 ? NC : 256);  // W_dkv rows per TMA box
   static constexpr int kABytes = kBM * kBK * 2;
-  static constexpr int kBBytes = N * kBK * 2;
+  // rows of a stage's weight region: in a cluster every CTA takes the widest
+  // slice's layout, so that multicast copies and barriers sit at the same
+  // offsets in all of them
+  static constexpr int kBRows = CL > 1 ? 64 + DR : N;
+  static constexpr int kBBytes = kBRows * kBK * 2;
+  static constexpr int kTxBytes = kABytes + N * kBK * 2;  // lands in this CTA per stage
+  static constexpr int kXParts = CL == 3 ? 2 : CL;       // ranks fetching a part of each x box
+  static constexpr int kXRows = kBM / kXParts;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBarBytes = 256;
-  static constexpr int kFit = (232448 - 1024 - kBarBytes) / kStageBytes;
+  // [CL][128] partial sums of squares at the front of shared memory: the same
+  // offset in every CTA of a cluster, whichever slice it computes
+  static constexpr int kRedOff = CL > 1 ? (CL * kBM * 4 + 1023) / 1024 * 1024 : 0;
+  static constexpr int kFit = (232448 - 1024 - kBarBytes - kRedOff) / kStageBytes;
   static constexpr int kStages = kFit > 6 ? 6 : kFit;
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
+  static constexpr int kSmemBytes = 1024 + kRedOff + kStages * kStageBytes + kBarBytes;
   static constexpr uint32_t kTmemCols = N <= 32 ? 32 : (N <= 64 ? 64 : (N <= 256 ? 256 : 512));
   // output staging row: N bf16 plus 16 bytes, so rows start on different banks
   static constexpr int kOutStride = N * 2 + 16;
   static_assert(kBM * kOutStride + kBM * 8 <= kStages * kStageBytes, "staging fits in the ring");
   static_assert(DC % 32 == 0 && DR % 32 == 0 && DR <= 64 && (DC <= 256 || DC % 256 == 0),
                 "shape");
-  static_assert(PART == kPartBoth || DC > 256, "parts are split only when d_c > 256");
+  static_assert(N > 0 && NC % 32 == 0 && (NK == 0 || NK == DR), "parts");
+  static_assert((NC == DC && NK == DR && CL == 1) || (DC > 256 && CL == 1) ||
+                    (CL == DC / 64 && CL >= 2 && DC <= 256 && NC == 64),
+                "parts are split for d_c > 256, or over a cluster of 64-column slices");
   static_assert(N <= 512, "accumulator must fit in TMEM");
-  static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
+  static_assert(kStageBytes % 1024 == 0 && (kXRows * 128) % 1024 == 0, "swizzle-atom alignment");
+  static_assert(kXParts * kXRows == kBM && kWcBox > 0, "x box split over the cluster");
   static_assert(kStages >= 2, "smem");
 };
 
@@ -72,15 +92,18 @@ struct AppendKParams {
   int* status;
 };
 
-template <int DC, int DR, int PART>
+// tile: the token tile (128 tokens) of this CTA; c0: its first column of c
+template <int DC, int DR, int NC, int NK, int CL>
 __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUtensorMap* tm_wc,
-                                            const CUtensorMap* tm_wk, const AppendKParams& p) {
-  using S = AppendShape<DC, DR, PART>;
-  constexpr int NC = S::NC;
-  constexpr int NK = S::NK;
+                                            const CUtensorMap* tm_wk, const AppendKParams& p,
+                                            int tile, int c0) {
+  using S = AppendShape<DC, DR, NC, NK, CL>;
   constexpr int NST = S::kStages;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = align_smem_1024(smem_raw);
+  uint8_t* base = align_smem_1024(smem_raw);
+  // [CL][128] partial sums of squares, written by every CTA of the cluster
+  float* ss_all = reinterpret_cast<float*>(base);
+  uint8_t* smem = base + S::kRedOff;  // the stage ring
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NST * S::kStageBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + NST;
@@ -91,13 +114,13 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.y;
-  const int row0 = blockIdx.x * kBM;
+  const int row0 = tile * kBM;
   const WaitCtx wc{abort_flag, p.status};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < NST; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], CL);  // released by the MMA of every CTA of the cluster
     }
     mbar_init(acc_full, 1);
     *abort_flag = 0;
@@ -111,6 +134,10 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  constexpr uint16_t kAll = static_cast<uint16_t>((1u << CL) - 1u);
+  const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+  // every CTA's barriers must be initialised before a peer's multicast lands
+  if constexpr (CL > 1) cluster_sync();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -123,17 +150,36 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
         if (kb >= NST && !mbar_wait(&empty[st], ((kb / NST) - 1) & 1, wc)) break;
         uint8_t* a = smem + st * S::kStageBytes;
         uint8_t* bm = a + S::kABytes;
-        mbar_arrive_expect_tx(&full[st], S::kStageBytes);
-        tma_load_3d(a, tm_x, &full[st], kb * kBK, row0, b);
+        mbar_arrive_expect_tx(&full[st], S::kTxBytes);
+        if constexpr (CL > 1) {
+          // this rank's rows of the x box, multicast to every CTA of the cluster
+          if (crank < S::kXParts)
+            tma_load_3d_mc(a + crank * S::kXRows * 128, tm_x, &full[st], kb * kBK,
+                           row0 + crank * S::kXRows, b, kAll);
+        } else {
+          tma_load_3d(a, tm_x, &full[st], kb * kBK, row0, b);
+        }
         if constexpr (NC > 0)
           for (int h = 0; h < NC / S::kWcBox; ++h)
-            tma_load_2d(bm + h * S::kWcBox * 128, tm_wc, &full[st], kb * kBK, h * S::kWcBox);
+            tma_load_2d(bm + h * S::kWcBox * 128, tm_wc, &full[st], kb * kBK,
+                        c0 + h * S::kWcBox);
         if constexpr (NK > 0) tma_load_2d(bm + NC * 128, tm_wk, &full[st], kb * kBK, 0);
         issued = kb + 1;
+      }
+      if constexpr (CL > 1) {
+        // the peers' MMAs release every stage through this CTA's barriers:
+        // their last releases must have landed before the CTA may exit
+        for (int st = 0; st < NST && st < p.k_blocks && !*abort_flag; ++st)
+          mbar_wait(&empty[st], (((p.k_blocks - st + NST - 1) / NST) - 1) & 1, wc);
       }
       if (*abort_flag)
         for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
           mbar_wait_drain(&full[u % NST], (u / NST) & 1, p.status);
+    }
+    __syncwarp();
+    if constexpr (CL > 1) {  // the cluster's second barrier phase (see the epilogue)
+      cluster_arrive_release();
+      cluster_wait_acquire();
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -168,12 +214,19 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
             }
           }
         }
-        umma_commit(&empty[st]);
+        if constexpr (CL > 1)
+          umma_commit_mc(&empty[st], kAll);  // the stage's x part came from every rank
+        else
+          umma_commit(&empty[st]);
       }
       umma_commit(acc_full);
       if (!ok) mbar_wait_drain(acc_full, 0, p.status);
     }
     __syncwarp();
+    if constexpr (CL > 1) {  // the cluster's second barrier phase
+      cluster_arrive_release();
+      cluster_wait_acquire();
+    }
   } else {
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
@@ -187,10 +240,10 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     // pieces of a row instead of each thread writing its own row.
     uint8_t* stage_out = smem;                                   // [128][kOutStride]
     long long* slot_of = reinterpret_cast<long long*>(smem + kBM * S::kOutStride);  // [128]
+    // pass 1: sum of squares of this CTA's c columns (fp32)
+    float ss = 0.f;
     if (have_acc) {
       tc_fence_after();
-      // pass 1: mean square of c over d_c (fp32)
-      float ss = 0.f;
 #pragma unroll 1
       for (int cb = 0; cb < NC / 32; ++cb) {
         uint32_t v[32];
@@ -202,6 +255,20 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
           ss = fmaf(f, f, ss);
         }
       }
+    }
+    if constexpr (CL > 1) {
+      // every CTA pushes its row's partial sum into slot [its rank][row] of
+      // every CTA, then all threads of the cluster pass the second barrier
+      // phase (release / acquire), on every path, so that no CTA waits for
+      // one that left; after it the sums are read locally, in rank order
+      const uint32_t local = smem_u32(ss_all + (c0 / 64) * kBM + r);
+      for (int q = 0; q < CL; ++q) dsmem_st_f32(dsmem_addr(local, q), ss);
+      cluster_arrive_release();
+      cluster_wait_acquire();
+      ss = 0.f;
+      for (int q = 0; q < CL; ++q) ss += ss_all[q * kBM + r];
+    }
+    if (have_acc) {
       const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
       const long long f = p.first_frame + n / p.T;
       const long long slot = frame_base_slot(f, p.T, p.W, p.S) + n % p.T;
@@ -217,7 +284,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           uint4 g4 = make_uint4(0x3f803f80u, 0x3f803f80u, 0x3f803f80u, 0x3f803f80u);  // ones
-          if (p.gamma) g4 = __ldg(reinterpret_cast<const uint4*>(p.gamma + cb * 32) + i);
+          if (p.gamma) g4 = __ldg(reinterpret_cast<const uint4*>(p.gamma + c0 + cb * 32) + i);
           gw[4 * i] = g4.x; gw[4 * i + 1] = g4.y; gw[4 * i + 2] = g4.z; gw[4 * i + 3] = g4.w;
         }
         uint32_t pk[16];
@@ -276,7 +343,8 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
         if (slot < 0) continue;
         const uint4 v = *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
         if (ch < kChunksC)
-          *reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC + ch * 8) = v;
+          *reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC + c0 +
+                                    ch * 8) = v;
         else
           *reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR +
                                     (ch - kChunksC) * 8) = v;
@@ -297,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mla_append_tc_kernel(const __grid_constant__ CUtensorMap tm_x,
                          const __grid_constant__ CUtensorMap tm_wc,
                          const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
-  append_body<DC, DR, kPartBoth>(&tm_x, &tm_wc, &tm_wk, p);
+  append_body<DC, DR, DC, DR, 1>(&tm_x, &tm_wc, &tm_wk, p, blockIdx.x, 0);
 }
 
 // d_c > 256: blockIdx.z = 0 computes c, 1 computes k^R, for the same tokens
@@ -307,32 +375,100 @@ __global__ void __launch_bounds__(kThreads, 1)
                                const __grid_constant__ CUtensorMap tm_wc,
                                const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
   if (blockIdx.z == 0)
-    append_body<DC, DR, kPartC>(&tm_x, &tm_wc, &tm_wk, p);
+    append_body<DC, DR, DC, 0, 1>(&tm_x, &tm_wc, &tm_wk, p, blockIdx.x, 0);
   else
-    append_body<DC, DR, kPartK>(&tm_x, &tm_wc, &tm_wk, p);
+    append_body<DC, DR, 0, DR, 1>(&tm_x, &tm_wc, &tm_wk, p, blockIdx.x, 0);
+}
+
+// Small grids: a cluster of d_c/64 CTAs per token tile; rank q computes c
+// columns [64q, 64q + 64), the last rank k^R as well.
+template <int DC, int DR>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_append_tc_cluster_kernel(const __grid_constant__ CUtensorMap tm_x,
+                                 const __grid_constant__ CUtensorMap tm_wc,
+                                 const __grid_constant__ CUtensorMap tm_wk,
+                                 const AppendKParams p) {
+  constexpr int CL = DC / 64;
+  const int q = static_cast<int>(cluster_ctarank());
+  const int tile = blockIdx.x / CL;
+  if (q < CL - 1)
+    append_body<DC, DR, 64, 0, CL>(&tm_x, &tm_wc, &tm_wk, p, tile, q * 64);
+  else
+    append_body<DC, DR, 64, DR, CL>(&tm_x, &tm_wc, &tm_wk, p, tile, q * 64);
 }
 
 template <int DC, int DR>
 int launch_tc(const AppendArgs& a) {
   constexpr bool kSplit = DC > 256;
-  using S = AppendShape<DC, DR, kSplit ? kPartC : kPartBoth>;
-  using SK = AppendShape<DC, DR, kSplit ? kPartK : kPartBoth>;
-  constexpr int kSmem = S::kSmemBytes > SK::kSmemBytes ? S::kSmemBytes : SK::kSmemBytes;
+  constexpr bool kClusterable = DC >= 128 && DC <= 256;
+  constexpr int kCl = kClusterable ? DC / 64 : 2;  // cluster size of the small-grid form
+  const int tiles = (a.n_tok + kBM - 1) / kBM;
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // the cluster form when its CTAs all fit in one wave (e.g. one Wan chunk at
+  // batch 1: 37 tiles x 3 = 111 CTAs) and every cluster is resident at once;
+  // otherwise one CTA per tile already fills the SMs and streaming the
+  // weights once per tile is the cheaper way
+  bool cluster = false;
+  if constexpr (kClusterable) {
+    const long long clusters = static_cast<long long>(tiles) * a.batch;
+    if (clusters * kCl <= sms) {
+      static int resident = -1;  // co-resident clusters of this shape (per process)
+      if (resident < 0) {
+        using SC0 = AppendShape<DC, DR, 64, 0, kCl>;
+        using SC1 = AppendShape<DC, DR, 64, DR, kCl>;
+        constexpr int kSm = SC0::kSmemBytes > SC1::kSmemBytes ? SC0::kSmemBytes : SC1::kSmemBytes;
+        auto kc = mla_append_tc_cluster_kernel<DC, DR>;
+        int n = 0;
+        cudaLaunchConfig_t oc = {};
+        oc.gridDim = dim3(kCl * static_cast<unsigned>(clusters), 1, 1);
+        oc.blockDim = dim3(kThreads, 1, 1);
+        oc.dynamicSmemBytes = kSm;
+        cudaLaunchAttribute oa[1];
+        oa[0].id = cudaLaunchAttributeClusterDimension;
+        oa[0].val.clusterDim.x = kCl;
+        oa[0].val.clusterDim.y = 1;
+        oa[0].val.clusterDim.z = 1;
+        oc.attrs = oa;
+        oc.numAttrs = 1;
+        if (cudaFuncSetAttribute(kc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSm) !=
+                cudaSuccess ||
+            cudaOccupancyMaxActiveClusters(&n, kc, &oc) != cudaSuccess) {
+          cudaGetLastError();  // a failed query only disables the cluster form
+          n = 0;
+        }
+        resident = n;
+      }
+      cluster = clusters <= resident;
+    }
+  }
+  // shapes of the CTAs each form launches (d_c > 256: the c and k^R halves;
+  // the cluster form: a 64-column c slice and k^R; else both parts)
+  using S = AppendShape<DC, DR, DC, kSplit ? 0 : DR>;
+  using SK = AppendShape<DC, DR, kSplit ? 0 : DC, DR>;
+  using SCc = std::conditional_t<kClusterable, AppendShape<DC, DR, 64, 0, kCl>, S>;
+  using SCk = std::conditional_t<kClusterable, AppendShape<DC, DR, 64, DR, kCl>, S>;
+  constexpr int kSmemPlain = S::kSmemBytes > SK::kSmemBytes ? S::kSmemBytes : SK::kSmemBytes;
+  constexpr int kSmemCl = SCc::kSmemBytes > SCk::kSmemBytes ? SCc::kSmemBytes : SCk::kSmemBytes;
+  const int smem = cluster ? kSmemCl : kSmemPlain;
   CUtensorMap tm_x, tm_wc, tm_wk;
   const unsigned long long H = a.hidden, n_tok = a.n_tok;
-  if (!encode_map_3d_bf16(&tm_x, a.x, H, n_tok, a.batch, H * 2, n_tok * H * 2, kBK, kBM,
-                          CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !encode_map_2d_bf16(&tm_wc, a.w_dkv, H, DC, H * 2, kBK, S::kWcBox,
+  if (!encode_map_3d_bf16(&tm_x, a.x, H, n_tok, a.batch, H * 2, n_tok * H * 2, kBK,
+                          cluster ? SCc::kXRows : kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_2d_bf16(&tm_wc, a.w_dkv, H, DC, H * 2, kBK, cluster ? 64 : S::kWcBox,
                           CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_wk, a.w_kr, H, DR, H * 2, kBK, DR, CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
-  auto kern = [] {
-    if constexpr (kSplit)
-      return mla_append_tc_split_kernel<DC, DR>;
-    else
-      return mla_append_tc_kernel<DC, DR>;
-  }();
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  using KernFn = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, AppendKParams);
+  KernFn kern;
+  if constexpr (kSplit)
+    kern = mla_append_tc_split_kernel<DC, DR>;
+  else if constexpr (kClusterable)
+    kern = cluster ? mla_append_tc_cluster_kernel<DC, DR> : mla_append_tc_kernel<DC, DR>;
+  else
+    kern = mla_append_tc_kernel<DC, DR>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return MLA_ERR_CUDA;
@@ -357,9 +493,20 @@ int launch_tc(const AppendArgs& a) {
   kp.use_rmsnorm = a.use_rmsnorm;
   kp.eps = a.eps;
   kp.status = a.status;
-  const dim3 grid((a.n_tok + kBM - 1) / kBM, a.batch, kSplit ? 2 : 1);
-  kern<<<grid, kThreads, kSmem, a.stream>>>(tm_x, tm_wc, tm_wk, kp);
-  e = cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(cluster ? tiles * kCl : tiles, a.batch, kSplit ? 2 : 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = a.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cluster ? kCl : 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, tm_x, tm_wc, tm_wk, kp);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return MLA_ERR_CUDA;
