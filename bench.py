@@ -84,6 +84,17 @@ def kernel_source_hash(name):
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
+def append_kernel_name(w):
+    """The append kernel the library launches for this shape: a cluster of
+    d_c/64 CTAs per token tile when those CTAs fit in one wave, else one CTA
+    per tile (the launch also checks that the clusters are co-resident)."""
+    tiles = -(-w.chunk_tokens // 128)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count if torch.cuda.is_available() else 152
+    if 128 <= w.d_c <= 256 and tiles * w.batch * (w.d_c // 64) <= sms:
+        return f"mla_append_tc_cluster_kernel<{w.d_c},{w.d_r}>"
+    return f"mla_append_tc_kernel<{w.d_c},{w.d_r}>"
+
+
 def profiled_traffic(summary, kernel_src):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
     the current kernel source (else None)."""
@@ -420,7 +431,7 @@ def run_ours(args, w, rank, world, local_rank):
                         if w.batch == 1 else None),
         },
         "roofline_append": {
-            "bound": "hbm", "kernel": "mla_append_tc_kernel<192,32>",
+            "bound": "hbm", "kernel": append_kernel_name(w),
             "algorithmic_bytes_per_launch": append_bytes(w),
             "achieved": append_bytes(w) / max(app_ms, 1e-6) / 1e6,
             "peak": peaks["hbm_gbs"], "unit": "GB/s",
