@@ -376,6 +376,128 @@ def test_rollout_positions_to_960():
     assert_close(f64(o).reshape(w.batch, -1, w.d_c)[:, rows], ref, what="rollout o_lat")
 
 
+# ------------------------------------------------------------ edge cases
+@pytest.mark.parametrize("d_c", [192, 512])
+def test_single_query_token(d_c):
+    """Nq = 1: 12 rows in one mostly empty row tile (a lone CTA, or the CTA
+    pair of the split-output instance at d_c = 512)."""
+    w = small(d_c=d_c, grid_h=6, grid_w=7, window_frames=3, batch=2)
+    cache, c, k = upload_cache(w, 61, 3)
+    q_c, q_r = synth.draw_queries(w, 1, 62)
+    q_pos = synth.grid_positions(w, 2, 1)[:, 5:6].contiguous()
+    o = torch.empty(w.batch, 1, w.heads, d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    assert_close(f64(o), oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid()),
+                 what=f"Nq=1 d_c={d_c}")
+
+
+def _chain(w, weights, chunks, q_first, q_n, seed):
+    """Append on both sides, then attend with the newest chunk's tokens."""
+    cache, oc = run_chunks(w, weights, chunks, seed=seed)
+    nq = q_n * w.tokens_per_frame
+    q_c, q_r = synth.draw_queries(w, nq, seed + 50)
+    q_pos = synth.grid_positions(w, q_first, q_n)
+    o = torch.empty(w.batch, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    valid = oc.valid_slots()
+    ref = np.stack([O.latent_attention(f64(q_c[b]), f64(q_r[b]), q_pos[b].numpy(),
+                                       oc.c[b, valid], oc.kr[b, valid], w.head_dim, spec_of(w))
+                    for b in range(w.batch)])
+    return f64(o), ref
+
+
+def test_single_key_window():
+    """One token per frame and a one-frame window: a single valid key (the
+    rest of its 128-key block masked); the append's token tile holds one
+    token and 127 rows past the end."""
+    w = small(grid_h=1, grid_w=1, window_frames=1, batch=2)
+    weights = synth.draw_layer_weights(w, seed=63)
+    got, ref = _chain(w, weights, [(0, 1), (1, 1), (2, 1)], 2, 1, 640)
+    assert_close(got, ref, what="single key")
+
+
+def test_one_frame_window_overwritten():
+    """W = 1: every chunk overwrites the whole ring; the current chunk is
+    rewritten once more before attention."""
+    w = small(grid_h=6, grid_w=6, window_frames=1, batch=2)
+    weights = synth.draw_layer_weights(w, seed=65)
+    got, ref = _chain(w, weights, [(0, 1), (1, 1), (2, 1), (2, 1)], 2, 1, 660)
+    assert_close(got, ref, what="W=1")
+
+
+def test_positions_at_table_end():
+    """Key and query coordinates at the last row of the RoPE table (1023) on
+    every axis, next to coordinates at 0."""
+    w = small(grid_h=4, grid_w=4, window_frames=2, batch=1)
+    assert w.rope_table_len == 1024
+    weights = synth.draw_layer_weights(w, seed=67)
+    cfg = V.make_config(w)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    oc = O.OracleCache(w.batch, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r)
+    dev = {k: v.cuda() for k, v in weights.items()}
+    T = w.tokens_per_frame
+    for f in range(2):
+        x = synth.draw_tokens(w, T, 680 + f)
+        pos = synth.grid_positions(w, f, 1)
+        pos[:, :, 0] = 1022 + f
+        pos[:, ::2, 1:] = 1023 - pos[:, ::2, 1:]     # half the tokens at the top rows
+        V.mla_cache_append(cache, x.cuda(), dev["w_dkv"], dev["gamma_kv"], dev["w_kr"],
+                           pos.cuda(), f, 1)
+        O.cache_append(oc, f64(x), f64(weights["w_dkv"]), f64(weights["w_kr"]), pos.numpy(),
+                       f, 1, gamma=f64(weights["gamma_kv"]), eps=w.rms_eps, spec=spec_of(w))
+    q_c, q_r = synth.draw_queries(w, T, 690)
+    q_pos = synth.grid_positions(w, 1, 1)
+    q_pos[:, :, 0] = 1023
+    q_pos[:, 1::2, 1:] = 1023 - q_pos[:, 1::2, 1:]
+    o = torch.empty(w.batch, T, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    valid = oc.valid_slots()
+    assert_close(f64(cache.c)[:, valid], oc.c[:, valid], what="c at table end")
+    assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what="k_rope at table end")
+    ref = O.latent_attention(f64(q_c[0]), f64(q_r[0]), q_pos[0].numpy(), oc.c[0, valid],
+                             oc.kr[0, valid], w.head_dim, spec_of(w))
+    assert_close(f64(o)[0], ref, what="attention at table end")
+
+
+def test_cluster_and_per_tile_append_forms_agree():
+    """The Wan chunk at batch 1 takes the cluster form of the append (37
+    clusters of 3 CTAs, each 64 columns of c); at batch 2 (222 CTAs would
+    exceed one wave) one CTA per token tile computes all 224 columns. The
+    same activations give the same cache rows up to one bf16 rounding step
+    (the cluster form adds the RMSNorm sum up in three partial sums)."""
+    w1 = synth.workload("wan")
+    w2 = w1.with_(batch=2)
+    weights = {k: v.cuda() for k, v in synth.draw_layer_weights(w1, 69).items()}
+    x1 = synth.draw_tokens(w1, w1.chunk_tokens, 70)
+    x2 = torch.cat([x1, synth.draw_tokens(w1, w1.chunk_tokens, 71)], 0)
+    out = []
+    for w, x in ((w1, x1), (w2, x2)):
+        cache = V.LatentCache(V.make_config(w))
+        V.mla_cache_reset(cache)
+        pos = synth.grid_positions(w, 0, w.chunk_frames).cuda()
+        V.mla_cache_append(cache, x.cuda(), weights["w_dkv"], weights["gamma_kv"],
+                           weights["w_kr"], pos, 0, w.chunk_frames)
+        torch.cuda.synchronize()
+        n = w.chunk_tokens
+        out.append((cache.c[0, :n].float().cpu(), cache.kr[0, :n].float().cpu()))
+    (c1, k1), (c2, k2) = out
+    for a, b_, name in ((c1, c2, "c"), (k1, k2, "k^R")):
+        assert torch.all((a - b_).abs() <= 2.0 ** -7 * b_.abs() + 1e-6), f"{name}: beyond 1 ulp"
+    # and both against the oracle on sampled tokens
+    rows = np.random.default_rng(2).choice(w1.chunk_tokens, 24, replace=False)
+    xs = f64(x1)[0, rows]
+    pos = synth.grid_positions(w1, 0, w1.chunk_frames)[0, rows].numpy()
+    oc = O.OracleCache(1, len(rows), 1, w1.d_c, w1.d_r)
+    O.cache_append(oc, xs[None], f64(weights["w_dkv"].cpu()), f64(weights["w_kr"].cpu()), pos[None],
+                   0, 1, gamma=f64(weights["gamma_kv"].cpu()), eps=w1.rms_eps, spec=spec_of(w1))
+    assert_close(c1.numpy()[rows], oc.c[0], what="cluster-form c")
+    assert_close(k1.numpy()[rows], oc.kr[0], what="cluster-form k_rope")
+
+
 # ------------------------------------------------------------ error paths
 def test_position_out_of_table_sets_device_status():
     w = small()

@@ -152,6 +152,20 @@ def test_sink_window_other_latent_sizes(d_c, d_r, pairs, dims):
     assert_close(f64(o), oracle_window(w, oc, q_c, q_r, q_pos), what=f"window o_lat {d_c}/{d_r}")
 
 
+def test_sink_window_with_one_fifo_slot():
+    """S = W - 1: two sink frames and a FIFO of one frame, rolled to frame 8."""
+    w = synth.workload("tiny", window_frames=3, sink_frames=2, batch=2)
+    weights = synth.draw_layer_weights(w, seed=89)
+    chunks = [(f, 1) for f in range(9)]
+    cache, oc = window_chunks(w, weights, chunks)
+    assert oc.held_frames() == [0, 1, 8]
+    T = w.tokens_per_frame
+    q_c, q_r = synth.draw_queries(w, T, 90)
+    q_pos = synth.grid_positions(w, 8, 1)
+    o = window_forward(w, cache, q_c, q_r, q_pos)
+    assert_close(f64(o), oracle_window(w, oc, q_c, q_r, q_pos), what="S = W - 1")
+
+
 def test_contiguous_window_matches_rotate_at_append_path():
     """No sink: re-indexed rotate-at-use attention equals the rotate-at-append
     hot path on the same inputs (RoPE relativity), after the ring wrapped."""
