@@ -1,6 +1,7 @@
 // Plain SIMT kernels for the same two calls: no tensor cores, no TMA, fp32
 // arithmetic throughout. They are the debug reference on the device (selected
-// with MLA_FLAG_SIMT) and cover shapes the tcgen05 kernels do not (d_c = 512).
+// with MLA_FLAG_SIMT) and cover shapes the tcgen05 kernels do not (d_c or d_r
+// outside {64, 128, 192, 256, 512} x {32, 64}).
 // Same equations as the tensor-core path: Eq. (ckv), App. D.2 RMSNorm,
 // Eq. (krope), App. D.4 ring slot; Eq. (score) and App. E latent output.
 #include <cmath>
