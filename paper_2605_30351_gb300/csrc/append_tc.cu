@@ -16,6 +16,9 @@
 // TMEM columns; the launch then runs two CTAs per token tile (blockIdx.z):
 // one accumulates c (two N = 256 MMAs per K step) and applies RMSNorm, the
 // other accumulates k^R and applies RoPE. Both stream the same x tile.
+// When one CTA per token tile would leave most SMs idle (one chunk at batch
+// 1), a cluster of d_c/64 CTAs shares each token tile, one per 64 columns of
+// c (see AppendShape).
 #include <cmath>
 #include <type_traits>
 
