@@ -2,8 +2,10 @@
 // the query prologue (Eqs. cq, qnope, qrope with App. E's absorbed weights)
 // and the output projection (Eq. absorb-v). C[M x N] = A[M x K] B[N x K]^T,
 // both operands K-major, fp32 accumulation, one 128 x BN tile per CTA:
-//   warp 0     TMA producer (A [128 x 64], B [BN x 64] per stage, SW128)
-//   warp 1     TMEM allocation; one lane issues tcgen05.mma (N = BN)
+//   warp 0     TMA producer (A [128 x 64], B [BN x 64] per stage, SW128;
+//              B in two boxes when BN > 256)
+//   warp 1     TMEM allocation; one lane issues tcgen05.mma (N = BN, or two
+//              MMAs of N = BN/2 when BN > 256)
 //   warps 2-5  epilogue, thread i = row i: TMEM -> registers -> bf16 staged
 //              in shared memory, then stored by all 128 threads together.
 // Epilogues:
@@ -38,9 +40,11 @@ struct GemmShape {
   static constexpr int kStages = kFit > MAXST ? MAXST : kFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
   static constexpr int kOutStride = BN * 2 + 16;  // staged bf16 row + 16 bytes (bank spread)
-  static constexpr uint32_t kTmemCols = BN <= 128 ? 128 : 256;
-  static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN, false, false);
-  static_assert(BN % 32 == 0 && BN <= 256, "tile width");
+  static constexpr uint32_t kTmemCols = BN <= 128 ? 128 : (BN <= 256 ? 256 : 512);
+  static constexpr int kHalves = BN > 256 ? 2 : 1;  // MMAs (and B boxes) per K step
+  static constexpr int kBN1 = BN / kHalves;         // columns of one MMA / rows of one B box
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN1, false, false);
+  static_assert(BN % 32 == 0 && BN <= 512 && kBN1 % 32 == 0, "tile width");
   static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
   static_assert(kBM * kOutStride <= kStages * kStageBytes, "staging fits in the ring");
 };
@@ -107,7 +111,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint8_t* a = smem + st * S::kStageBytes;
         mbar_arrive_expect_tx(&full[st], S::kStageBytes);
         tma_load_2d(a, &tm_a, &full[st], kb * kBK, m0);
-        tma_load_2d(a + S::kABytes, &tm_b, &full[st], kb * kBK, n0);
+#pragma unroll
+        for (int h = 0; h < S::kHalves; ++h)
+          tma_load_2d(a + S::kABytes + h * S::kBN1 * 128, &tm_b, &full[st], kb * kBK,
+                      n0 + h * S::kBN1);
         issued = kb + 1;
       }
       if (*abort_flag)
@@ -129,8 +136,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ba = aa + S::kABytes;
 #pragma unroll
         for (int k = 0; k < kBK / 16; ++k)
-          umma_ss(tmem, sdesc(aa + k * 32, 16, 1024, kSw128), sdesc(ba + k * 32, 16, 1024, kSw128),
-                  S::kIdesc, (kb | k) != 0 ? 1u : 0u);
+#pragma unroll
+          for (int h = 0; h < S::kHalves; ++h)
+            umma_ss(tmem + h * S::kBN1, sdesc(aa + k * 32, 16, 1024, kSw128),
+                    sdesc(ba + h * S::kBN1 * 128 + k * 32, 16, 1024, kSw128), S::kIdesc,
+                    (kb | k) != 0 ? 1u : 0u);
         umma_commit(&empty[st]);
       }
       umma_commit(acc_full);
@@ -212,7 +222,7 @@ int launch_gemm(const void* a, const void* b, int M, int N, int K, GemmKParams k
   if (K % kBK != 0 || N % 8 != 0) return MLA_ERR_UNSUPPORTED;
   CUtensorMap tm_a, tm_b;
   if (!encode_map_2d_bf16(&tm_a, a, K, M, K * 2ull, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-      !encode_map_2d_bf16(&tm_b, b, K, N, K * 2ull, kBK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+      !encode_map_2d_bf16(&tm_b, b, K, N, K * 2ull, kBK, S::kBN1, CU_TENSOR_MAP_SWIZZLE_128B))
     return MLA_ERR_CUDA;
   auto kern = mla_gemm_tc_kernel<BN, EPI, MAXST>;
   cudaError_t e =
@@ -377,13 +387,19 @@ int launch_output_projection(const OutProjArgs& a) {
   k.c = static_cast<__nv_bfloat16*>(a.y);
   k.ldc = a.hidden;
   k.status = a.status;
-  // Two CTAs per SM (two-stage ring). 192-wide tiles when 256-wide ones would
-  // leave the GPU less than two CTAs per SM (one Wan chunk: 29 vs 35 us);
-  // 256-wide otherwise (four chunks: 100 vs 119 us).
+  // 384-wide tiles, one CTA per SM with three 64 KB stages, when they fit in
+  // one wave (one Wan chunk: 37 x 4 = 148 CTAs); otherwise two CTAs per SM
+  // (two-stage ring): 192-wide tiles when 256-wide ones would leave the GPU
+  // less than two CTAs per SM (one chunk: 29 vs 35 us), 256-wide otherwise
+  // (four chunks: 100 vs 119 us).
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const long long ctas256 = static_cast<long long>((a.rows + kBM - 1) / kBM) * ((a.hidden + 255) / 256);
+  const long long row_tiles = (a.rows + kBM - 1) / kBM;
+  if (a.hidden % 384 == 0 && row_tiles * (a.hidden / 384) <= sms)
+    return launch_gemm<384, kStore, 3>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
+                                       a.stream);
+  const long long ctas256 = row_tiles * ((a.hidden + 255) / 256);
   if (ctas256 < 2ll * sms && a.hidden % 192 == 0)
     return launch_gemm<192, kStore, 2>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
                                        a.stream);
