@@ -200,6 +200,35 @@ def test_attention_dc512_simt():
     assert_close(f64(o), oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid()), what="d_c=512")
 
 
+# the append's two forms at every latent size with a tensor-core instance:
+# small grids take clusters of d_c/64 CTAs (2, 3 or 4; x multicast in 64- or
+# 32-row parts), larger ones one CTA per token tile
+APPEND_SIZES = [(64, 32, (6, 5, 5), (44, 42, 42)), (128, 32, (6, 5, 5), (44, 42, 42)),
+                (256, 32, (6, 5, 5), (44, 42, 42)), (64, 64, (12, 10, 10), (64, 64, 64)),
+                (128, 64, (12, 10, 10), (64, 64, 64)), (256, 64, (12, 10, 10), (64, 64, 64))]
+
+
+@pytest.mark.parametrize("d_c,d_r,pairs,dims", APPEND_SIZES)
+@pytest.mark.parametrize("form", ["small", "large"])
+def test_append_latent_sizes(d_c, d_r, pairs, dims, form):
+    """small: T = 100, batch 2, ring wrap (3 token tiles per chunk: the
+    cluster form for d_c >= 128); large: the Wan grid, 3-frame chunks,
+    batch 3 (111 token tiles: one CTA per tile)."""
+    if form == "small":
+        w = small(d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims, grid_h=10, grid_w=10,
+                  window_frames=5, batch=2)
+        chunks = [(0, 3), (3, 3), (3, 3), (6, 2)]
+    else:
+        w = synth.workload("wan").with_(d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims,
+                                        window_frames=6, batch=3)
+        chunks = [(0, 3), (3, 3), (6, 3)]
+    weights = synth.draw_layer_weights(w, seed=23 + d_c + d_r)
+    cache, oc = run_chunks(w, weights, chunks, seed=230)
+    valid = oc.valid_slots()
+    assert_close(f64(cache.c)[:, valid], oc.c[:, valid], what=f"c {d_c}/{d_r} {form}")
+    assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what=f"k_rope {d_c}/{d_r} {form}")
+
+
 # d_c = 512: the attention output is split over a CTA pair (256 columns
 # each) and the append runs its c and k^R halves in separate CTAs
 DC512 = [(32, (6, 5, 5), (44, 42, 42)), (64, (12, 10, 10), (64, 64, 64))]
