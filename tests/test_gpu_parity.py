@@ -345,6 +345,31 @@ def test_attention_wan_sampled_rows():
     assert_close(got, ref, what="wan sampled")
 
 
+@pytest.mark.parametrize("d_c,d_r,pairs,dims", [
+    (64, 32, (6, 5, 5), (44, 42, 42)), (128, 32, (6, 5, 5), (44, 42, 42)),
+    (256, 32, (6, 5, 5), (44, 42, 42)), (64, 64, (12, 10, 10), (64, 64, 64)),
+    (128, 64, (12, 10, 10), (64, 64, 64)), (192, 64, (12, 10, 10), (64, 64, 64)),
+    (256, 64, (12, 10, 10), (64, 64, 64)),
+])
+def test_attention_latent_sizes_wan_sampled_rows(d_c, d_r, pairs, dims):
+    """Every tensor-core instance at the Wan shape (32,760 keys: the stage
+    ring laps many times), oracle on sampled rows of the first, a middle and
+    the last row tile."""
+    w = synth.workload("wan").with_(d_c=d_c, d_r=d_r, rope_pairs=pairs, rope_axis_dims=dims)
+    cache, c, k = upload_cache(w, 41 + d_c + d_r, w.window_frames)
+    q_c, q_r = synth.draw_queries(w, w.chunk_tokens, 42 + d_c)
+    q_pos = synth.grid_positions(w, 18, 3)
+    o = torch.empty(1, w.chunk_tokens, w.heads, d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), q_pos.cuda(), o)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(d_c + d_r)
+    n = w.chunk_tokens * w.heads
+    rows = np.unique(np.concatenate([[0, 127, n // 2, n - 1], rng.choice(n, 20, replace=False)]))
+    ref = oracle_latent(w, q_c, q_r, q_pos, c, k, cache.n_valid(), rows=rows)
+    got = f64(o).reshape(1, -1, d_c)[:, rows]
+    assert_close(got, ref, what=f"Wan rows d_c={d_c} d_r={d_r}")
+
+
 def test_append_then_attention_chain():
     """Each side runs its own append then attention: end-to-end latent output."""
     w = small(grid_h=10, grid_w=12, window_frames=4, chunk_frames=2, batch=2)
