@@ -526,6 +526,9 @@ def run_sweep(args, rank):
             ms = time_launches(lambda: V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o,
                                                                stream), steps, 2, stream)
             fl = flops_per_layer(w)[0]
+            if kind == "tcgen05" and d_c > 256:
+                # the output is split over a CTA pair and both CTAs score the full key tile
+                kind = "tcgen05 (output split over a CTA pair; score computed by both)"
             rows.append({
                 "layout": "mla", "d_c": d_c, "d_r": d_r, "kernel": kind,
                 "bytes_per_token_per_layer": 2 * (d_c + d_r),
@@ -533,7 +536,10 @@ def run_sweep(args, rank):
                 "compression_vs_dense": 2 * w.heads * w.head_dim / (d_c + d_r),
                 "ms_per_chunk_layer": ms, "tflops": fl / (ms * 1e-3) / 1e12,
                 "frac_of_measured_bf16_burst": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"],
-                "flop_per_row_key": 4 * d_c + 2 * d_r})
+                "flop_per_row_key": 4 * d_c + 2 * d_r,
+                **({"issued_flop_per_row_key": 4 * (d_c + d_r) + 2 * d_c,
+                    "issued_tflops": fl / (4 * d_c + 2 * d_r) * (4 * (d_c + d_r) + 2 * d_c)
+                    / (ms * 1e-3) / 1e12} if d_c > 256 else {})})
             del s
             torch.cuda.empty_cache()
     # dense per-head baseline: q, k, v with d_h = 128, 12 heads, same window
