@@ -1,8 +1,9 @@
 """Helper run in a subprocess by test_gpu_debug_build.py: loads the library
 named on the command line (release or debug build), runs a fixed set of
 calls (append + attention on the 21-frame ring, the sink window, the
-decompression, the query prologue and output projection) on seeded inputs
-and saves every output plus the device status word."""
+decompression, the query prologue and output projection; the append's
+cluster and split forms and the split-output attention at d_c = 256 and 512)
+on seeded inputs and saves every output plus the device status word."""
 
 import os
 import sys
@@ -59,6 +60,25 @@ def main(lib_path, out_path):
             out["q_c"], out["q_r"], out["y"] = qc2.cpu(), qr2.cpu(), y.cpu()
         torch.cuda.synchronize()
         out[f"c{sink}"], out[f"kr{sink}"], out[f"o{sink}"] = cache.c.cpu(), cache.kr.cpu(), o.cpu()
+    # the other launch forms: a cluster of 4 CTAs per token tile (d_c = 256) and
+    # the split append and split-output attention of d_c = 512
+    for d_c in (256, 512):
+        w = synth.workload("tiny", grid_h=10, grid_w=10, window_frames=3, batch=2, d_c=d_c,
+                           rope_pairs=(6, 5, 5))
+        wt = {k: t.cuda() for k, t in synth.draw_layer_weights(w, 33).items()}
+        cache = V.LatentCache(V.make_config(w))
+        V.mla_cache_reset(cache)
+        T = w.tokens_per_frame
+        for f in range(4):
+            x = synth.draw_tokens(w, T, 70 + f).cuda()
+            V.mla_cache_append(cache, x, wt["w_dkv"], wt["gamma_kv"], wt["w_kr"],
+                               synth.grid_positions(w, f, 1).cuda(), f, 1)
+        q_c, q_r = synth.draw_queries(w, T, 80)
+        o = torch.empty(w.batch, T, w.heads, d_c, dtype=torch.bfloat16, device="cuda")
+        V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(), synth.grid_positions(w, 3, 1).cuda(),
+                                o)
+        torch.cuda.synchronize()
+        out[f"c_{d_c}"], out[f"kr_{d_c}"], out[f"o_{d_c}"] = cache.c.cpu(), cache.kr.cpu(), o.cpu()
     out["status"] = V.mla_device_status(clear=True)
     torch.save(out, out_path)
 
