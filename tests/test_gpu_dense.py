@@ -102,6 +102,27 @@ def test_decompress_reconstructs_per_head_keys_and_values(name, kw, slots_checke
         assert torch.equal(rope_bits[:, h], src)
 
 
+@pytest.mark.parametrize("d_c,d_r,pairs", [(64, 32, (6, 5, 5)), (128, 32, (6, 5, 5)),
+                                        (256, 32, (6, 5, 5)), (128, 64, (12, 10, 10)),
+                                        (256, 64, (12, 10, 10))])
+def test_decompress_other_latent_sizes(d_c, d_r, pairs):
+    """The decompression's other instances on a ragged 500-slot window, batch 2."""
+    w = synth.workload("tiny", grid_h=10, grid_w=10, window_frames=5, batch=2, d_c=d_c, d_r=d_r,
+                       rope_pairs=pairs)
+    wt = synth.draw_layer_weights(w, seed=63 + d_c + d_r)
+    cache, c, kr = _upload_cache(w, 64 + d_c)
+    k, v = _decompress(w, cache, wt)
+    dn = w.head_dim - w.d_r
+    k_nope = np.einsum("hec,bjc->bhje", f64(wt["w_uk"]), c)
+    v_ref = np.einsum("hvc,bjc->bhjv", f64(wt["w_uv"]), c)
+    assert_close(f64(k[..., :dn]), k_nope, what=f"k_nope d_c={d_c} d_r={d_r}")
+    assert_close(f64(v), v_ref, what=f"v d_c={d_c} d_r={d_r}")
+    rope_bits = k[..., dn:].cpu().view(torch.int16)
+    src = cache.kr.cpu().view(torch.int16)
+    for h in range(w.heads):
+        assert torch.equal(rope_bits[:, h], src)
+
+
 def test_decompress_then_dense_matches_non_absorbed_oracle():
     """x -> GPU append -> decompress -> dense attention with per-head queries
     [q^nope | RoPE(q^R)], against the oracle's non-absorbed forward (Sec. 3.3)."""
