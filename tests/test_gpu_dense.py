@@ -33,12 +33,13 @@ def draw_dense(w, nq, slots, seed):
     return q, k, v
 
 
-@pytest.mark.parametrize("nq,slots,n_valid,batch", [
-    (64, 256, 256, 1),     # the tiny config's shape
-    (300, 500, 387, 2),    # ragged tiles and a partially valid window
+@pytest.mark.parametrize("nq,slots,n_valid,batch,head_dim", [
+    (64, 256, 256, 1, 128),     # the tiny config's shape
+    (300, 500, 387, 2, 128),    # ragged tiles and a partially valid window
+    (300, 500, 387, 2, 64),     # the d_h = 64 instance
 ])
-def test_dense_attention_matches_oracle(nq, slots, n_valid, batch):
-    w = synth.workload("tiny", batch=batch)
+def test_dense_attention_matches_oracle(nq, slots, n_valid, batch, head_dim):
+    w = synth.workload("tiny", batch=batch, head_dim=head_dim)
     q, k, v = draw_dense(w, nq, slots, 17)
     o = torch.empty_like(q, device="cuda")
     V.mla_dense_attention_forward(V.make_config(w), q.cuda(), k.cuda(), v.cuda(), n_valid, o)

@@ -136,6 +136,9 @@ def test_sink_window_attention_parity(case, flags):
 
 @pytest.mark.parametrize("d_c,d_r,pairs,dims", [(128, 64, (12, 10, 10), (64, 64, 64)),
                                                (64, 32, (6, 5, 5), (44, 42, 42)),
+                                               (192, 64, (12, 10, 10), (64, 64, 64)),
+                                               (256, 32, (6, 5, 5), (44, 42, 42)),
+                                               (256, 64, (12, 10, 10), (64, 64, 64)),
                                                (512, 32, (6, 5, 5), (44, 42, 42))])
 def test_sink_window_other_latent_sizes(d_c, d_r, pairs, dims):
     """The window path at other (d_c, d_r): the assembly kernel's 16-byte
