@@ -49,7 +49,8 @@ extern "C" {
  *  head_dim        d_h = d_nope + d_rope (128); the score is divided by
  *                  sqrt(head_dim) (Eq. score)
  *  d_c             width of the shared KV latent c^KV (192)   (Eq. ckv)
- *  d_r             width of the shared positional key k^R (32) (Eq. krope)
+ *  d_r             width of the shared positional key k^R (32) (Eq. krope);
+ *                  positive (the decoupled key always exists on this path)
  *  d_q             width of the query latent c^Q (768), used by the query prologue
  *  rope_pairs_*    complex pairs per axis; 2*(t+h+w) must equal d_r (App. D.3)
  *  rope_dim_*      band width D_a of each axis: pair i of axis a rotates with

@@ -60,7 +60,7 @@ int axis_dim(const mla_config& c, int a) {
 
 int check_config(const mla_config* c) {
   if (!c) return MLA_ERR_ARG;
-  if (c->hidden <= 0 || c->heads <= 0 || c->head_dim <= 0 || c->d_c <= 0 || c->d_r < 0 ||
+  if (c->hidden <= 0 || c->heads <= 0 || c->head_dim <= 0 || c->d_c <= 0 || c->d_r <= 0 ||
       c->tokens_per_frame <= 0 || c->window_frames <= 0 || c->batch <= 0 ||
       c->rope_table_len <= 0 || !(c->rope_theta > 0.0) || !(c->rms_eps >= 0.f))
     return MLA_ERR_ARG;

@@ -58,6 +58,10 @@ def test_config_validation():
     bad.window_frames = 0
     assert V.mla_config_check(bad) == V.MLA_ERR_ARG
     bad = V.make_config(w)
+    bad.d_r = 0                               # no positional key (and no RoPE pairs)
+    bad.rope_pairs_t = bad.rope_pairs_h = bad.rope_pairs_w = 0
+    assert V.mla_config_check(bad) == V.MLA_ERR_ARG
+    bad = V.make_config(w)
     bad.sink_frames = w.window_frames         # no frame slot left for the FIFO part
     assert V.mla_config_check(bad) == V.MLA_ERR_ARG
     bad.sink_frames = -1
