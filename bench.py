@@ -393,6 +393,14 @@ def run_ours(args, w, rank, world, local_rank):
     attn_ms_mean = statistics.fmean(attn_ms)
     achieved = attn_l / (attn_ms_mean * 1e-3) / 1e12
     app_ms = statistics.fmean(app_ms_l)
+    # the burst peak for a kernel timed over a short region, the sustained one
+    # (a seconds-long loop under the power cap) once the timed region is that long
+    if ms_max >= 1000.0:
+        peak, peak_kind = peaks["bf16_tflops_sustained"], "sustained"
+        peak_why = f"timed region {ms_max / 1e3:.1f} s"
+    else:
+        peak, peak_kind = peaks["bf16_tflops"], "burst"
+        peak_why = f"timed region {ms_max:.0f} ms"
     out = {
         "metric": METRIC,
         "value": whole_job_throughput(attn_fl + app_fl, ms_step, world),
@@ -420,10 +428,11 @@ def run_ours(args, w, rank, world, local_rank):
         "attention_ms": attn_ms_mean,
         "append_ms": app_ms,
         "roofline": {
-            "bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"],
-            "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"],
+            "bound": "tensor", "achieved": achieved, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak,
+            "frac_of_burst": achieved / peaks["bf16_tflops"],
             "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
-            "peak_source": f"{peaks['source']} bf16 dense (burst)",
+            "peak_source": f"{peaks['source']} bf16 dense ({peak_kind}: {peak_why})",
             "kernel": ("window_assemble_kernel + mla_attn_tc_kernel<192,32,2,128> (events around both)"
                        if w.sink_frames else "mla_attn_tc_kernel<192,32,2,128>"),
             "algorithmic_flops_per_launch": attn_l,

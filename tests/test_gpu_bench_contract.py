@@ -57,6 +57,9 @@ def test_roofline_object(line):
     assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
     assert abs(r["frac"] - r["achieved"] / r["peak"]) < 1e-6
     assert 0.3 < r["frac"] < 1.6
+    # a short timed region is compared with the burst peak (the sustained one
+    # applies once the region runs for seconds under the power cap)
+    assert "burst" in r["peak_source"] and abs(r["frac"] - r["frac_of_burst"]) < 1e-9
 
 
 def test_cpu_baseline_object(line):
