@@ -148,3 +148,53 @@ def test_sink_window_before_eviction_is_absolute():
     ref = O.latent_attention(q_c, q_r, q_pos, rot.c[0, valid], rot.kr[0, valid], 8, SPEC)
     np.testing.assert_allclose(O.window_attention(raw, 0, q_c, q_r, q_pos, 8, SPEC), ref,
                                rtol=0, atol=1e-12)
+
+
+def test_window_attention_matches_brute_force_loops():
+    """Pure-Python loops, independent of the oracle's vectorised code: the held
+    frames are numbered by hand, every pair is rotated with explicit cos/sin at
+    (local t, h, w), and the softmax is summed term by term."""
+    import math
+    spec = O.RopeSpec(pairs=(2, 1, 0), axis_dims=(4, 2, 2), theta=10000.0)
+    T, W, S, dc, d = 2, 3, 1, 2, 5
+    rng = np.random.default_rng(11)
+    cache = O.OracleCache(1, T, W, dc, spec.d_r, sink_frames=S)
+    w_dkv = rng.standard_normal((dc, d))
+    w_kr = rng.standard_normal((spec.d_r, d))
+    for f in range(6):
+        x = rng.standard_normal((1, T, d))
+        pos = np.array([[[f, k, 0] for k in range(T)]])
+        O.cache_append(cache, x, w_dkv, w_kr, pos, f, 1)
+    q_c = rng.standard_normal((3, 1, dc))
+    q_r = rng.standard_normal((3, 1, spec.d_r))
+    q_pos = np.array([[5, 0, 0], [5, 1, 0], [4, 1, 0]])
+    got = O.window_attention(cache, 0, q_c, q_r, q_pos, 4, spec)
+
+    held = [0, 4, 5]                         # the sink, then the two newest frames
+    local = {f: i for i, f in enumerate(held)}
+    bands = [(0, 0), (0, 1), (1, 0)]         # (axis, index within the axis) per pair
+
+    def rotate(v, pos):
+        out = []
+        for p, (a, i) in enumerate(bands):
+            ang = pos[a] * spec.theta ** (-2.0 * i / spec.axis_dims[a])
+            x0, x1 = v[2 * p], v[2 * p + 1]
+            out += [x0 * math.cos(ang) - x1 * math.sin(ang), x0 * math.sin(ang) + x1 * math.cos(ang)]
+        return out
+
+    keys = []
+    for s in range(W * T):
+        f = int(cache.frame_of_slot[s])
+        if f in local:
+            h = int(cache.pos_of_slot[0, s, 1])
+            keys.append((list(cache.c[0, s]), rotate(list(cache.kr[0, s]), (local[f], h, 0))))
+    assert len(keys) == 3 * T
+    for n in range(3):
+        qr = rotate(list(q_r[n, 0]), (local[int(q_pos[n, 0])], int(q_pos[n, 1]), 0))
+        scores = [(sum(q_c[n, 0, i] * c[i] for i in range(dc)) +
+                   sum(qr[i] * k[i] for i in range(spec.d_r))) / 2.0 for c, k in keys]
+        mx = max(scores)
+        e = [math.exp(sc - mx) for sc in scores]
+        z = sum(e)
+        o = [sum(e[j] / z * keys[j][0][i] for j in range(len(keys))) for i in range(dc)]
+        np.testing.assert_allclose(got[n, 0], o, rtol=0, atol=1e-12)
