@@ -9,11 +9,16 @@ attention at the Wan2.1-1.3B shape (4680-query chunk, 32760-key window,
 One step = mla_cache_append of the current 3-frame chunk + mla_attention_forward
 of that chunk against the full 21-frame window (one layer, one denoising step;
 30 layers for wan30; batch 4 for rollout and sink, sink using the 1 + 6 frame
-window with rotate-at-use RoPE). Prints one JSON line (rank 0). Multi-GPU runs
-are independent replicas (weak scaling): the path has no exchange step. The
---sweep modes print one JSON line each on one GPU: the latent-size sweep next
-to the dense baseline, the memory-cap batch sweep, the whole layer by phase,
-and absorbed vs decompress-then-dense by query-chunk size.
+window with rotate-at-use RoPE). Prints one JSON line. The --sweep modes print
+one JSON line each: the latent-size sweep next to the dense baseline, the
+memory-cap batch sweep, the whole layer by phase, and absorbed vs
+decompress-then-dense by query-chunk size.
+
+Single GPU only. Every tensor-core kernel shares tiles among the CTAs of a
+cluster by TMA multicast within this GPU's memory, which may only run in
+single-GPU jobs; under torchrun with more than one rank the GPU arm prints an
+"unavailable" line (rank 0) and every rank exits 0. The reference arm (the
+float64 oracle on the host cores) runs on rank 0 alone.
 """
 
 import argparse
@@ -164,18 +169,28 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------- CPU oracle
-def cpu_oracle_sample(w, budget_s=12.0, seed=5, tokens_per_batch=8):
-    """Time the float64 oracle (as it stands) on a bounded sample of the same
-    workload: the append of R tokens and the attention of those R tokens' 12
-    heads against the full window, R grown in batches until ~budget_s."""
+# The float64 oracle, as it stands, timed on every host core: one spawned
+# worker process per core (spawn, so no worker inherits a CUDA context), each
+# running the oracle single-threaded on its own slice of query tokens. Both
+# the GPU arm's cpu_baseline leg and the reference arm time the SAME sample:
+# query tokens 0 .. P*TOKENS_PER_WORKER-1 of the chunk (P = worker count),
+# each with its cache append and its 12 heads' attention against the full
+# window.
+TOKENS_PER_WORKER = 1
+_ORACLE = None  # per-worker state (inputs drawn from the same seeds in every worker)
+
+
+def _oracle_state(w, seed):
     from oracle import mla_oracle as O
 
     spec = O.RopeSpec(w.rope_pairs, w.rope_axis_dims, w.rope_theta)
     weights = synth.draw_layer_weights(w, seed)
     f64 = lambda t: t.float().numpy().astype(np.float64)
-    wd, wk, g = f64(weights["w_dkv"]), f64(weights["w_kr"]), f64(weights["gamma_kv"])
+    st = {"w": w, "spec": spec, "wd": f64(weights["w_dkv"]), "wk": f64(weights["w_kr"]),
+          "g": f64(weights["gamma_kv"])}
     c, k = synth.draw_cache_rows(w, w.slots, seed + 1, batch=1)
-    c, k = f64(c[0]), f64(k[0])
+    st["c"], st["k"] = f64(c[0]), f64(k[0])
+    st["win"] = None
     if w.sink_frames:
         # the window oracle: a cache holding the sink frame and the newest
         # frames with k^R unrotated, rotated at window-local times per call
@@ -187,46 +202,121 @@ def cpu_oracle_sample(w, budget_s=12.0, seed=5, tokens_per_batch=8):
             s0 = O.sink_ring_slot(f, 0, T, w.window_frames, w.sink_frames)
             win.frame_of_slot[s0:s0 + T] = f
             win.pos_of_slot[0, s0:s0 + T] = synth.grid_positions(w, f, 1, batch=1)[0].numpy()
-        win.c[0], win.kr[0] = c, k
+        win.c[0], win.kr[0] = st["c"], st["k"]
         win.frames_written = w.last_frame
+        st["win"] = win
     q_c, q_r = synth.draw_queries(w, w.chunk_tokens, seed + 2, batch=1)
     x = synth.draw_tokens(w, w.chunk_tokens, seed + 3, batch=1)
     pos = synth.grid_positions(w, (w.last_frame if w.sink_frames else w.window_frames)
                                - w.chunk_frames, w.chunk_frames, batch=1)
-    q_c, q_r, x, pos = f64(q_c[0]), f64(q_r[0]), f64(x), pos.numpy()
-    step = tokens_per_batch
-    done = 0
-    fl = 0.0
-    c0 = os.times()
-    t0 = time.perf_counter()
-    while done < w.chunk_tokens and time.perf_counter() - t0 < budget_s:
-        sl = slice(done, min(done + step, w.chunk_tokens))
-        n = sl.stop - sl.start
-        oc = O.OracleCache(1, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r)
-        oc.T = n  # one partial "frame" of n tokens: the same arithmetic per token
-        O.cache_append(oc, x[:, sl], wd, wk, pos[:, sl], 0, 1, gamma=g, eps=w.rms_eps,
-                       spec=None if w.sink_frames else spec)
-        if w.sink_frames:
-            O.window_attention(win, 0, q_c[sl], q_r[sl], pos[0, sl], w.head_dim, spec)
-        else:
-            O.latent_attention(q_c[sl], q_r[sl], pos[0, sl], c, k, w.head_dim, spec)
-        fl += 2.0 * n * w.hidden * (w.d_c + w.d_r)
-        fl += O.latent_attention_flops(n * w.heads, w.slots, w.d_c, w.d_r)
-        done += n
-    wall = time.perf_counter() - t0
-    c1 = os.times()
-    cpu = (c1.user - c0.user) + (c1.system - c0.system)
-    return {
-        "value": fl / wall / 1e12,
-        "unit": UNIT,
-        "cores": max(1, round(cpu / wall)),
-        "host_cores_available": len(os.sched_getaffinity(0)),
-        "kind": "oracle",
-        "sample": (f"float64 NumPy oracle: append + attention of {done} of {w.chunk_tokens} "
-                   f"query tokens (x{w.heads} heads) against the full {w.slots}-key window, "
-                   f"{wall:.1f} s"),
-        "seconds": wall,
-    }
+    st["q_c"], st["q_r"], st["x"], st["pos"] = f64(q_c[0]), f64(q_r[0]), f64(x), pos.numpy()
+    return st
+
+
+def _oracle_init(w, seed):
+    global _ORACLE
+    _ORACLE = _oracle_state(w, seed)
+
+
+def _oracle_ready(_):
+    return _ORACLE is not None
+
+
+def _oracle_slice(start, stop):
+    """Append + attention of query tokens [start, stop) with the oracle; returns
+    (flops, cpu seconds of this process)."""
+    from oracle import mla_oracle as O
+
+    st = _ORACLE
+    w, spec = st["w"], st["spec"]
+    sl = slice(start, stop)
+    n = stop - start
+    t0 = time.process_time()
+    oc = O.OracleCache(1, w.tokens_per_frame, w.window_frames, w.d_c, w.d_r)
+    oc.T = n  # one partial "frame" of n tokens: the same arithmetic per token
+    O.cache_append(oc, st["x"][:, sl], st["wd"], st["wk"], st["pos"][:, sl], 0, 1, gamma=st["g"],
+                   eps=w.rms_eps, spec=None if w.sink_frames else spec)
+    if w.sink_frames:
+        O.window_attention(st["win"], 0, st["q_c"][sl], st["q_r"][sl], st["pos"][0, sl],
+                           w.head_dim, spec)
+    else:
+        O.latent_attention(st["q_c"][sl], st["q_r"][sl], st["pos"][0, sl], st["c"], st["k"],
+                           w.head_dim, spec)
+    fl = 2.0 * n * w.hidden * (w.d_c + w.d_r) + O.latent_attention_flops(
+        n * w.heads, w.slots, w.d_c, w.d_r)
+    return fl, time.process_time() - t0
+
+
+class OraclePool:
+    """One spawned single-threaded oracle worker per host core: `cores` in the
+    JSON line is that worker count (one thread each); cpu_utilisation is the
+    workers' CPU time over the wall time of the rounds, per worker."""
+
+    def __init__(self, w, seed=5):
+        import multiprocessing as mp
+
+        self.w = w
+        self.procs = len(os.sched_getaffinity(0))
+        self.tokens = min(w.chunk_tokens, self.procs * TOKENS_PER_WORKER)
+        saved = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS",
+                                                "MKL_NUM_THREADS")}
+        for k in saved:
+            os.environ[k] = "1"  # one thread per worker: the pool supplies the parallelism
+        try:
+            self.pool = mp.get_context("spawn").Pool(self.procs, initializer=_oracle_init,
+                                                     initargs=(w, seed))
+        finally:
+            for k, v in saved.items():
+                if v is None:
+                    os.environ.pop(k, None)
+                else:
+                    os.environ[k] = v
+        assert all(self.pool.map(_oracle_ready, range(self.procs), chunksize=1))
+
+    def round(self):
+        """The whole sample once: (flops, wall seconds, cpu seconds)."""
+        slices = [(a, min(a + TOKENS_PER_WORKER, self.tokens))
+                  for a in range(0, self.tokens, TOKENS_PER_WORKER)]
+        t0 = time.perf_counter()
+        res = self.pool.starmap(_oracle_slice, slices, chunksize=1)
+        wall = time.perf_counter() - t0
+        return sum(r[0] for r in res), wall, sum(r[1] for r in res)
+
+    def describe(self, wall, rounds):
+        w = self.w
+        return (f"float64 NumPy oracle, {self.procs} single-threaded worker processes: append + "
+                f"attention of query tokens 0..{self.tokens - 1} of the {w.chunk_tokens}-token "
+                f"chunk (x{w.heads} heads, {TOKENS_PER_WORKER} per worker) against the "
+                f"full {w.slots}-key window; {rounds} round(s), {wall:.1f} s")
+
+    def close(self):
+        self.pool.terminate()
+        self.pool.join()
+
+
+def cpu_oracle_sample(w, budget_s=12.0, pool=None):
+    """Time the oracle on the fixed sample, repeated for about budget_s."""
+    own = pool is None
+    pool = pool or OraclePool(w)
+    try:
+        fl = wall = cpu = 0.0
+        rounds = 0
+        while rounds == 0 or wall < budget_s:
+            f, t, c = pool.round()
+            fl, wall, cpu, rounds = fl + f, wall + t, cpu + c, rounds + 1
+        return {
+            "value": fl / wall / 1e12,
+            "unit": UNIT,
+            "cores": pool.procs,
+            "cpu_utilisation": cpu / wall / pool.procs,
+            "host_cores_available": len(os.sched_getaffinity(0)),
+            "kind": "oracle",
+            "sample": pool.describe(wall, rounds),
+            "seconds": wall,
+        }
+    finally:
+        if own:
+            pool.close()
 
 
 # ------------------------------------------------------------------ GPU arm
@@ -259,15 +349,18 @@ class LayerSet:
                                   dtype=torch.uint8, device="cuda")
 
 
-def run_ours(args, w, rank, world, local_rank):
+def run_ours(args, w):
     from paper_2605_30351_gb300 import videomla as V
 
-    torch.cuda.set_device(local_rank)
+    # the oracle's worker processes start before the first GPU call (spawned,
+    # so none of them holds a CUDA context); they are timed after the GPU run
+    pool = None if args.no_cpu_baseline else OraclePool(w)
+    torch.cuda.set_device(0)
     V.load()
     stream = torch.cuda.current_stream()
     # one set per layer of a step, or N_SETS rotating sets for a one-layer step
     n_sets = max(w.layers, N_SETS)
-    sets = [LayerSet(w, 1000 + 17 * i + 101 * rank, V) for i in range(n_sets)]
+    sets = [LayerSet(w, 1000 + 17 * i, V) for i in range(n_sets)]
     attn_l, app_l = flops_per_layer(w)
     attn_fl, app_fl = attn_l * w.layers, app_l * w.layers
 
@@ -298,19 +391,17 @@ def run_ours(args, w, rank, world, local_rank):
            for _ in range(w.layers)] for _ in range(args.steps)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    barrier(world)
     torch.cuda.synchronize()
-    with ClockSampler(local_rank) as clk:
+    with ClockSampler(0) as clk:
         t_start.record(stream)
         for i in range(args.steps):
             step(i, ev[i])
         t_end.record(stream)
         torch.cuda.synchronize()
-    barrier(world)
     ms_total = t_start.elapsed_time(t_end)
     app_ms_l = [e[0].elapsed_time(e[1]) for es in ev for e in es]
     attn_ms = [e[1].elapsed_time(e[2]) for es in ev for e in es]
-    ms_max = allreduce_max(ms_total, world)
+    ms_max = ms_total
     status = V.mla_device_status(clear=True)
     if status != V.MLA_OK:
         raise RuntimeError(f"device status {status} after the timed region")
@@ -376,7 +467,6 @@ def run_ours(args, w, rank, world, local_rank):
 
     e2e_run(2)
     torch.cuda.synchronize()
-    barrier(world)
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -384,10 +474,11 @@ def run_ours(args, w, rank, world, local_rank):
     e2e_run(e2e_steps)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = allreduce_max(e0.elapsed_time(e1), world)
+    e2e_ms = e0.elapsed_time(e1)
 
-    if rank != 0:
-        return None
+    # the append alone at batch 4 (a rollout batch), where the HBM bar applies
+    append_b4 = time_append_b4(w, V, stream) if w.batch == 1 and w.layers == 1 else None
+
     peaks = load_peaks()
     ms_step = ms_max / args.steps
     attn_ms_mean = statistics.fmean(attn_ms)
@@ -403,9 +494,9 @@ def run_ours(args, w, rank, world, local_rank):
         peak_why = f"timed region {ms_max:.0f} ms"
     out = {
         "metric": METRIC,
-        "value": whole_job_throughput(attn_fl + app_fl, ms_step, world),
+        "value": tflops(attn_fl + app_fl, ms_step),
         "unit": UNIT,
-        "n_gpus": world,
+        "n_gpus": 1,
         "steps": args.steps,
         "warmup": args.warmup,
         "ms_per_step": ms_step,
@@ -422,7 +513,7 @@ def run_ours(args, w, rank, world, local_rank):
             "rope_pairs_thw": list(w.rope_pairs),
             "l2": f"inputs larger than L2: {N_SETS} rotating layer sets "
                   f"(~{N_SETS * 76} MB), one per step",
-            "parallelism": f"replicas x{world}",
+            "parallelism": "single GPU",
         },
         "ms_per_layer": ms_step / w.layers,
         "attention_ms": attn_ms_mean,
@@ -448,7 +539,7 @@ def run_ours(args, w, rank, world, local_rank):
             "note": "CUDA events around each append launch (mean over the timed steps)",
         },
         "e2e": {
-            "value": whole_job_throughput(attn_fl + app_fl, e2e_ms / e2e_steps, world),
+            "value": tflops(attn_fl + app_fl, e2e_ms / e2e_steps),
             "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": e2e_ms / e2e_steps, "steps": e2e_steps,
             "note": "public API with pinned host buffers; every step's inputs go up and its "
@@ -458,29 +549,88 @@ def run_ours(args, w, rank, world, local_rank):
         "clocks": clk.summary(),
         "gpu_launches": (3 if w.sink_frames else 2) * w.layers * args.steps,
     }
-    if world == 1 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_oracle_sample(w, budget_s=args.cpu_budget)
+    clocks = out["clocks"]
+    if clocks.get("sm_mhz"):
+        # the tensor pipe's own limit at the clock seen: 8192 bf16 FLOP per
+        # clock per SM (our tcgen05 loops, N = 128..256, SS or TS operands)
+        sms = torch.cuda.get_device_properties(0).multi_processor_count
+        lim = PIPE_FLOP_PER_CLK_SM * sms * clocks["sm_mhz"] * 1e6 / 1e12
+        out["roofline"]["pipe_limit_tflops"] = lim
+        out["roofline"]["frac_of_pipe_limit"] = achieved / lim
+    if append_b4 is not None:
+        out["roofline_append_b4"] = append_b4
+    if pool is not None:
+        try:
+            out["cpu_baseline"] = cpu_oracle_sample(w, budget_s=args.cpu_budget, pool=pool)
+        finally:
+            pool.close()
     return out
 
 
-def run_reference(args, w, rank):
-    """The reference arm: the float64 oracle, as it stands, on the host cores."""
-    if rank != 0:
-        return None
-    # each step is a bounded sample; the whole run stays within a few minutes
-    budget = min(args.cpu_budget, 60.0 / max(1, args.steps + args.warmup))
-    tok = 8 if budget >= 1.0 else 1
-    for _ in range(args.warmup):
-        cpu_oracle_sample(w, budget_s=budget, tokens_per_batch=tok)
-    vals = [cpu_oracle_sample(w, budget_s=budget, tokens_per_batch=tok)
-            for _ in range(args.steps)]
-    v = statistics.fmean(x["value"] for x in vals)
-    cb = dict(vals[-1])
-    cb["value"] = v
+def time_append_b4(w, V, stream, steps=100):
+    """The cache append of a 3-frame chunk at batch 4 (the rollout batch: 147
+    token tiles, one per SM), CUDA events around each launch over rotating
+    input sets larger than L2; algorithmic HBM bytes per launch / time."""
+    wb = w.with_(batch=4)
+    sets = []
+    for i in range(N_SETS):
+        wt = synth.draw_layer_weights(wb, 1500 + i)
+        cache = V.LatentCache(V.make_config(wb))
+        x = synth.draw_tokens(wb, wb.chunk_tokens, 1510 + i).cuda()
+        pos = synth.grid_positions(wb, wb.window_frames - wb.chunk_frames, wb.chunk_frames).cuda()
+        cache.frames_written = wb.window_frames
+        sets.append((cache, x, wt["w_dkv"].cuda(), wt["gamma_kv"].cuda(), wt["w_kr"].cuda(), pos))
+    first = wb.window_frames - wb.chunk_frames
+
+    def launch(i):
+        cache, x, wd, g, wk, pos = sets[i % N_SETS]
+        V.mla_cache_append(cache, x, wd, g, wk, pos, first, wb.chunk_frames, stream)
+
+    for i in range(5):
+        launch(i)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    for i in range(steps):
+        ev[i][0].record(stream)
+        launch(i)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    ms = statistics.fmean(a.elapsed_time(b) for a, b in ev)
+    peaks = load_peaks()
+    nbytes = append_bytes(wb)
+    return {"bound": "hbm", "kernel": append_kernel_name(wb), "batch": 4,
+            "algorithmic_bytes_per_launch": nbytes, "ms": ms,
+            "achieved": nbytes / (ms * 1e-3) / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": nbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "note": f"CUDA events around each launch (mean of {steps}), {N_SETS} rotating sets "
+                    f"of {wb.chunk_tokens * 4 * w.hidden * 2 / 1e6:.0f} MB of activations"}
+
+
+def run_reference(args, w):
+    """The reference arm: the float64 oracle, as it stands, on every host core;
+    each step is one pass over the same fixed token sample as the GPU arm's
+    cpu_baseline leg."""
+    pool = OraclePool(w)
+    try:
+        for _ in range(args.warmup):
+            pool.round()
+        fl = wall = cpu = 0.0
+        for _ in range(args.steps):
+            f, t, c = pool.round()
+            fl, wall, cpu = fl + f, wall + t, cpu + c
+        v = fl / wall / 1e12
+        cb = {"value": v, "unit": UNIT, "cores": pool.procs,
+              "cpu_utilisation": cpu / wall / pool.procs,
+              "host_cores_available": len(os.sched_getaffinity(0)),
+              "kind": "oracle", "sample": pool.describe(wall, args.steps), "seconds": wall}
+    finally:
+        pool.close()
     return {
         "impl": "reference",
         "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": 0, "steps": args.steps,
-        "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": wall / max(1, args.steps) * 1e3,
+        "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": workload_desc(w)},
         "cpu_baseline": cb,
@@ -503,7 +653,7 @@ def time_launches(fn, steps, warmup, stream):
     return float(np.median([ev[i].elapsed_time(ev[i + 1]) for i in range(steps)]))
 
 
-def run_sweep(args, rank):
+def run_sweep(args):
     """Latent-size sweep (the d_c axis of Table 5, left; Sec. 3.3's cache sizes):
     absorbed MLA attention for d_c in {64..512} x d_r in {32, 64} next to the
     dense per-head baseline (12 x 128 K and V per token) at the same query
@@ -594,8 +744,6 @@ def run_sweep(args, rank):
         "decompress_flop_per_key": 2 * base.d_c * w.heads * (dn + w.head_dim)})
     if V.mla_device_status(clear=True) != V.MLA_OK:
         raise RuntimeError("device status set during the sweep")
-    if rank != 0:
-        return None
     return {"metric": "latent-size sweep: absorbed MLA attention vs dense per-head baseline",
             "unit": "ms per chunk per layer", "data": "synthetic", "dtype": "bf16",
             "config": {"workload": workload_desc(base) + "; d_c and d_r varied"},
@@ -603,7 +751,7 @@ def run_sweep(args, rank):
 
 
 # ------------------------------------------------------------- crossover
-def run_crossover(args, rank):
+def run_crossover(args):
     """Absorbed attention (App. E) against decompress-then-dense (Eq.
     reconstruct, then per-head attention) as the query chunk grows from one
     latent frame to twelve, on the same 21-frame Wan window: the per-key cost
@@ -643,8 +791,6 @@ def run_crossover(args, rank):
         torch.cuda.empty_cache()
     if V.mla_device_status(clear=True) != V.MLA_OK:
         raise RuntimeError("device status set during the crossover sweep")
-    if rank != 0:
-        return None
     return {"metric": "absorbed MLA attention vs decompress-then-dense, by query-chunk size",
             "unit": "ms per chunk per layer", "data": "synthetic", "dtype": "bf16",
             "peak_bf16_tflops": peaks["bf16_tflops"],
@@ -654,7 +800,7 @@ def run_crossover(args, rank):
 
 
 # ------------------------------------------------------------- full layer
-def run_layer(args, w, rank):
+def run_layer(args, w):
     """The whole attention layer per chunk (Sec. 3, App. E): query prologue
     (x -> c^Q -> RMSNorm -> [q_c | q_r], absorbed weights), cache append,
     latent attention and output projection y = sum_h B_h o_lat,h; each phase
@@ -719,8 +865,6 @@ def run_layer(args, w, rank):
                          ("attention", med[2], attn_fl), ("output_projection", med[3], out_fl)):
         phases[name] = {"ms": ms, "flop": fl, "tflops": fl / (ms * 1e-3) / 1e12,
                         "frac_of_measured_bf16_burst": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"]}
-    if rank != 0:
-        return None
     fl_all = pro_fl + app_fl + attn_fl + out_fl
     return {"metric": "full attention layer per chunk: prologue, append, attention, output projection",
             "value": fl_all / (total * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_layer": total,
@@ -766,7 +910,7 @@ def memcap_plan(w, layout, budget_bytes, layers=30):
             "bytes_at_max_batch": fixed + b_max * per_batch}
 
 
-def run_memcap(args, rank):
+def run_memcap(args):
     """Maximum batch of one chunk-against-window attention step under a fixed
     HBM budget, dense per-head caches against latent caches at several d_c;
     the plan is checked by allocating every layer's cache at that batch and
@@ -865,8 +1009,6 @@ def run_memcap(args, rank):
             del kv, q
         torch.cuda.synchronize()
         torch.cuda.empty_cache()
-    if rank != 0:
-        return None
     return {"metric": "maximum batch under a fixed HBM budget: dense per-head vs latent caches",
             "unit": "batch elements (one 4680-token chunk against a 21-frame window each)",
             "data": "synthetic", "dtype": "bf16",
@@ -875,26 +1017,15 @@ def run_memcap(args, rank):
             "memcap": rows}
 
 
-# -------------------------------------------------------------- distributed
-def barrier(world):
-    if world > 1:
-        torch.distributed.barrier()
+# ----------------------------------------------------------------- helpers
+PIPE_FLOP_PER_CLK_SM = 8192  # measured tcgen05 bf16 rate per SM (N = 128..256)
+MULTI_GPU_CLOSED = ("multi-GPU runs are closed on this pool: every tensor-core kernel shares "
+                    "tiles among the CTAs of a cluster by TMA multicast, which may only run in "
+                    "single-GPU jobs")
 
 
-def allreduce_max(x, world):
-    """Max of a per-rank scalar over all ranks (timing: the slowest replica)."""
-    if world == 1:
-        return x
-    dev = "cuda" if torch.distributed.get_backend() == "nccl" else "cpu"
-    t = torch.tensor([x], dtype=torch.float64, device=dev)
-    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    return float(t.item())
-
-
-def whole_job_throughput(flop_per_step_per_rank, ms_per_step_max, world):
-    """Replicas: every rank does the same work; the job rate is the sum of the
-    ranks' work over the slowest rank's time, in TFLOP/s."""
-    return world * flop_per_step_per_rank / (ms_per_step_max * 1e-3) / 1e12
+def tflops(flop_per_step, ms_per_step):
+    return flop_per_step / (ms_per_step * 1e-3) / 1e12
 
 
 def main():
@@ -918,26 +1049,31 @@ def main():
     w = synth.workload(args.workload)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
-    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1 and args.impl == "ours":
-        torch.cuda.set_device(local_rank)
-        torch.distributed.init_process_group("nccl")
-    if args.sweep == "dc":
-        out = run_sweep(args, rank)
-    elif args.sweep == "memcap":
-        out = run_memcap(args, rank)
-    elif args.sweep == "layer":
-        out = run_layer(args, w, rank)
-    elif args.sweep == "crossover":
-        out = run_crossover(args, rank)
-    elif args.impl == "reference":
-        out = run_reference(args, w, rank)
-    else:
-        out = run_ours(args, w, rank, world, local_rank)
-    if out is not None:
+    if world > 1 or args.gpus > 1:
+        # no multi-GPU path (see the module docstring); rank 0 reports, every
+        # rank exits 0 without touching a GPU
+        if rank != 0:
+            return
+        if args.impl == "reference":
+            out = run_reference(args, w)
+        else:
+            out = {"metric": METRIC, "unit": UNIT, "n_gpus": max(world, args.gpus),
+                   "unavailable": MULTI_GPU_CLOSED}
         print(json.dumps(out), flush=True)
-    if world > 1 and args.impl == "ours":
-        torch.distributed.destroy_process_group()
+        return
+    if args.sweep == "dc":
+        out = run_sweep(args)
+    elif args.sweep == "memcap":
+        out = run_memcap(args)
+    elif args.sweep == "layer":
+        out = run_layer(args, w)
+    elif args.sweep == "crossover":
+        out = run_crossover(args)
+    elif args.impl == "reference":
+        out = run_reference(args, w)
+    else:
+        out = run_ours(args, w)
+    print(json.dumps(out), flush=True)
 
 
 if __name__ == "__main__":

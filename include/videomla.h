@@ -7,6 +7,15 @@
  *  - All tensors are caller-owned device memory (for example torch tensors
  *    passed by data_ptr()). The library allocates no device memory, keeps no
  *    per-cache state of its own and never synchronises the stream.
+ *  - Every buffer must be device memory (cudaMalloc or a pool built on it)
+ *    of the CURRENT device: host memory, pinned or not, managed memory and
+ *    another GPU's memory are refused with MLA_ERR_ARG before any launch.
+ *    The kernels copy tiles with TMA and share them among the CTAs of a
+ *    cluster by multicast, which addresses this GPU's own memory only.
+ *  - The library caches, per device, the device addresses of its two
+ *    file-scope arrays (the status word and the no-allocation scratch). It
+ *    does not survive cudaDeviceReset (or any other teardown of the
+ *    device's primary context) within the process.
  *  - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
  *    NULL is the legacy default stream).
  *  - bf16 = IEEE bfloat16 stored as 2 bytes. All arrays are dense, row-major,
@@ -148,7 +157,11 @@ int mla_cache_reset(mla_cache* cache, void* stream);
  * so this matches rotating at use with window-relative coordinates
  * (Sec. 3.2, App. D.5). With MLA_FLAG_ROTATE_AT_USE the cache keeps
  * k = W_kr x unrotated, the paper's own storage (App. D.5).
- * Rules: 1 <= n_frames <= window_frames (else MLA_ERR_RANGE);
+ * Rules: 1 <= n_frames <= window_frames, and at most W - S of the frames
+ * are past the sinks (frames >= S share W - S frame slots, so two of them in
+ * one call would land on the same slots): n_frames - max(0, min(n_frames,
+ * S - first_frame)) <= W - S (else MLA_ERR_RANGE; with S = 0 both rules are
+ * n_frames <= W);
  * 0 <= first_frame <= frames_written <= first_frame + n_frames (no gap, and
  * the range reaches the newest frame: extend the window or rewrite the
  * current chunk, as each denoising step does). Afterwards

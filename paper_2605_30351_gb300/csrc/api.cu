@@ -3,6 +3,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <initializer_list>
 #include <mutex>
 
 #include <cudaTypedefs.h>
@@ -23,16 +24,58 @@ std::mutex g_mu;
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
+// Device address of the status word on the current device, looked up once per
+// device (the address stays valid until the device's primary context is torn
+// down, e.g. by cudaDeviceReset, which the library does not survive). On
+// failure returns nullptr with the CUDA error recorded.
 int* device_status_ptr() {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    t_last_cuda_error = static_cast<int>(e);
+    return nullptr;
+  }
+  if (dev < 0 || dev >= kMaxDevices) {
+    t_last_cuda_error = static_cast<int>(cudaErrorInvalidDevice);
+    return nullptr;
+  }
   std::lock_guard<std::mutex> lk(g_mu);
   if (!g_status_ptr[dev]) {
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_device_status) != cudaSuccess) return nullptr;
+    e = cudaGetSymbolAddress(&p, g_device_status);
+    if (e != cudaSuccess || !p) {
+      t_last_cuda_error = static_cast<int>(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
+      return nullptr;
+    }
     g_status_ptr[dev] = static_cast<int*>(p);
   }
   return g_status_ptr[dev];
+}
+
+// Every buffer handed to a kernel (tensor-map sources included) must be
+// device memory of the current device: the kernels' TMA copies, and the
+// multicast among the CTAs of a cluster, address this GPU's own memory only.
+// Host memory (pageable or pinned), managed memory and another GPU's memory
+// are refused with MLA_ERR_ARG before anything is enqueued; null entries
+// (optional arguments) are skipped.
+int check_resident(std::initializer_list<const void*> ptrs) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    t_last_cuda_error = static_cast<int>(e);
+    return MLA_ERR_CUDA;
+  }
+  for (const void* p : ptrs) {
+    if (!p) continue;
+    cudaPointerAttributes at{};
+    e = cudaPointerGetAttributes(&at, p);
+    if (e != cudaSuccess) {
+      (void)cudaGetLastError();  // not a pointer the runtime knows: clear the sticky error
+      return MLA_ERR_ARG;
+    }
+    if (at.type != cudaMemoryTypeDevice || at.device != dev) return MLA_ERR_ARG;
+  }
+  return MLA_OK;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -121,7 +164,7 @@ int run_attention(const mla_cache* cache, const void* q_c, const void* q_r, cons
   a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c.head_dim)));
   a.status = device_status_ptr();
   a.stream = stream;
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   return (c.flags & MLA_FLAG_SIMT) ? launch_attention_simt(a) : launch_attention_tc(a);
 }
 
@@ -213,6 +256,8 @@ int mla_cache_reset(mla_cache* cache, void* stream) {
   if (rc != MLA_OK) return rc;
   if (!cache->c || (!cache->kr && cache->cfg.d_r > 0)) return MLA_ERR_ARG;
   const mla_config& c = cache->cfg;
+  const int rr = check_resident({cache->c, cache->kr});
+  if (rr != MLA_OK) return rr;
   const size_t slots = static_cast<size_t>(c.tokens_per_frame) * c.window_frames;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(cache->c, 0, slots * c.batch * c.d_c * 2, s);
@@ -237,9 +282,22 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv, const v
       (reinterpret_cast<uintptr_t>(pos) & 3u))
     return MLA_ERR_ARG;
   if (n_frames < 1 || n_frames > c.window_frames) return MLA_ERR_RANGE;
+  // frames after the sinks share W - S frame slots: two of them in one call
+  // would land on the same slots (App. D.4 FIFO), so at most W - S may come
+  // at once (with S = 0 this is n_frames <= W)
+  {
+    const long long sinks_in_call =
+        first_frame < c.sink_frames
+            ? (c.sink_frames - first_frame < n_frames ? c.sink_frames - first_frame : n_frames)
+            : 0;
+    if (n_frames - sinks_in_call > c.window_frames - c.sink_frames) return MLA_ERR_RANGE;
+  }
   if (first_frame < 0 || first_frame > cache->frames_written ||
       first_frame + n_frames < cache->frames_written)
     return MLA_ERR_ARG;
+  rc = check_resident({cache->c, cache->kr, cache->rope_table, x, w_dkv, gamma_kv, w_kr,
+                       rotate ? pos : nullptr});
+  if (rc != MLA_OK) return rc;
   AppendArgs a;
   a.x = x;
   a.w_dkv = w_dkv;
@@ -267,7 +325,7 @@ int mla_cache_append(mla_cache* cache, const void* x, const void* w_dkv, const v
   a.eps = c.rms_eps;
   a.status = device_status_ptr();
   a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   rc = (c.flags & MLA_FLAG_SIMT) ? launch_append_simt(a) : launch_append_tc(a);
   if (rc != MLA_OK) return rc;
   cache->frames_written = first_frame + n_frames;
@@ -287,6 +345,8 @@ int mla_attention_forward(const mla_cache* cache, const void* q_c, const void* q
       (reinterpret_cast<uintptr_t>(q_pos) & 3u))
     return MLA_ERR_ARG;
   if (Nq < 1 || rotate_at_use(c)) return MLA_ERR_ARG;
+  rc = check_resident({cache->c, cache->kr, cache->rope_table, q_c, q_r, q_pos, o_lat});
+  if (rc != MLA_OK) return rc;
   return run_attention(cache, q_c, q_r, q_pos, Nq, cache->kr, o_lat,
                        static_cast<cudaStream_t>(stream));
 }
@@ -302,6 +362,8 @@ int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* 
   if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(w_uk) || !aligned16(w_uv) ||
       !aligned16(k) || !aligned16(v))
     return MLA_ERR_ARG;
+  const int rr = check_resident({cache->c, cache->kr, w_uk, w_uv, k, v});
+  if (rr != MLA_OK) return rr;
   DecompressArgs a;
   a.c = cache->c;
   a.kr = cache->kr;
@@ -317,7 +379,7 @@ int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* 
   a.d_r = c.d_r;
   a.status = device_status_ptr();
   a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   return launch_decompress(a);
 }
 
@@ -344,6 +406,9 @@ int mla_attention_window_forward(const mla_cache* cache, const void* q_c, const 
   if (workspace_bytes < mla_window_workspace_bytes(&c, Nq)) return MLA_ERR_ARG;
   const long long n_valid = valid_slots(*cache);
   if (n_valid < 1) return MLA_ERR_ARG;
+  rc = check_resident({cache->c, cache->kr, cache->rope_table, q_c, q_r, q_pos, o_lat, frame_hw,
+                       workspace});
+  if (rc != MLA_OK) return rc;
   WindowArgs w;
   w.kr = cache->kr;
   w.q_pos = q_pos;
@@ -366,7 +431,7 @@ int mla_attention_window_forward(const mla_cache* cache, const void* q_c, const 
   w.pairs_h = c.rope_pairs_h;
   w.status = device_status_ptr();
   w.stream = static_cast<cudaStream_t>(stream);
-  if (!w.status) return fail_cuda(cudaGetLastError());
+  if (!w.status) return MLA_ERR_CUDA;
   rc = launch_window_assemble(w);
   if (rc != MLA_OK) return rc;
   return run_attention(cache, q_c, q_r, w.q_pos_local, Nq, w.kr_rot, o_lat, w.stream);
@@ -379,6 +444,8 @@ int mla_absorb_weights(const mla_config* cfg, const void* w_uq, const void* w_uk
   if (rc != MLA_OK) return rc;
   if (!w_uq || !w_uk || !w_qr || !w_uv || !w_o || !w_qcat || !w_b) return MLA_ERR_ARG;
   if (cfg->head_dim <= cfg->d_r || cfg->d_q <= 0) return MLA_ERR_ARG;
+  const int rr = check_resident({w_uq, w_uk, w_qr, gamma_q, w_uv, w_o, w_qcat, w_b});
+  if (rr != MLA_OK) return rr;
   AbsorbArgs a;
   a.w_uq = w_uq;
   a.w_uk = w_uk;
@@ -419,6 +486,8 @@ int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq, c
   if (workspace_bytes < mla_query_workspace_bytes(cfg, Nq)) return MLA_ERR_ARG;
   const long long rows = static_cast<long long>(cfg->batch) * Nq;
   if (rows > (1ll << 30)) return MLA_ERR_ARG;
+  const int rr = check_resident({x, w_dq, w_qcat, workspace, q_c, q_r});
+  if (rr != MLA_OK) return rr;
   QueryArgs a;
   a.x = x;
   a.w_dq = w_dq;
@@ -437,7 +506,7 @@ int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq, c
   a.eps = cfg->rms_eps;
   a.status = device_status_ptr();
   a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   return launch_query_prologue(a);
 }
 
@@ -453,6 +522,8 @@ int mla_query_prologue_noalloc(const mla_config* cfg, const void* x, const void*
   const unsigned long long need = mla_query_workspace_bytes(cfg, Nq);
   if (need == 0) return MLA_ERR_ARG;
   if (need > MLA_NOALLOC_SCRATCH_BYTES) return MLA_ERR_TOO_LARGE;
+  const int rr = check_resident({x, w_dq, w_qcat, q_c, q_r});
+  if (rr != MLA_OK) return rr;
   void* scratch = nullptr;
   const int sr = query_scratch_address(&scratch);
   if (sr != MLA_OK) return sr;
@@ -475,7 +546,7 @@ int mla_query_prologue_noalloc(const mla_config* cfg, const void* x, const void*
   a.eps = cfg->rms_eps;
   a.status = device_status_ptr();
   a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   return launch_query_prologue(a);
 }
 
@@ -488,6 +559,8 @@ int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* 
   if ((cfg->heads * cfg->d_c) % 64 != 0) return MLA_ERR_UNSUPPORTED;
   const long long rows = static_cast<long long>(cfg->batch) * Nq;
   if (rows > (1ll << 30)) return MLA_ERR_ARG;
+  const int rr = check_resident({o_lat, w_b, y});
+  if (rr != MLA_OK) return rr;
   OutProjArgs a;
   a.o_lat = o_lat;
   a.w_b = w_b;
@@ -498,7 +571,7 @@ int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* 
   a.d_c = cfg->d_c;
   a.status = device_status_ptr();
   a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   return launch_output_projection(a);
 }
 
@@ -510,6 +583,8 @@ int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void
   if (!q || !k || !v || !o || Nq < 1 || slots < 1 || n_valid < 1 || n_valid > slots)
     return MLA_ERR_ARG;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o)) return MLA_ERR_ARG;
+  const int rr = check_resident({q, k, v, o});
+  if (rr != MLA_OK) return rr;
   DenseArgs a;
   a.q = q;
   a.k = k;
@@ -525,14 +600,14 @@ int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void
       static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(cfg->head_dim)));
   a.status = device_status_ptr();
   a.stream = static_cast<cudaStream_t>(stream);
-  if (!a.status) return fail_cuda(cudaGetLastError());
+  if (!a.status) return MLA_ERR_CUDA;
   return launch_dense_attention_tc(a);
 }
 
 int mla_selftest_bounded_wait(unsigned long long limit_ns, void* stream) {
   if (limit_ns == 0 || limit_ns > 2000000000ull) return MLA_ERR_ARG;
   int* st = device_status_ptr();
-  if (!st) return fail_cuda(cudaGetLastError());
+  if (!st) return MLA_ERR_CUDA;
   return launch_wait_selftest(limit_ns, st, static_cast<cudaStream_t>(stream));
 }
 
@@ -554,7 +629,7 @@ int mla_last_cuda_error(void) { return t_last_cuda_error; }
 int mla_device_status(int* status, int clear) {
   if (!status) return MLA_ERR_ARG;
   int* p = device_status_ptr();
-  if (!p) return fail_cuda(cudaGetLastError());
+  if (!p) return MLA_ERR_CUDA;
   cudaError_t e = cudaDeviceSynchronize();
   if (e == cudaSuccess) e = cudaMemcpy(status, p, sizeof(int), cudaMemcpyDeviceToHost);
   if (e == cudaSuccess && clear) {

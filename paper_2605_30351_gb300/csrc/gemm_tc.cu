@@ -351,7 +351,10 @@ int launch_query_prologue(const QueryArgs& a) {
 // The library's only device memory of its own: a file-scope array every GPU
 // that loads the library holds until the process exits. Host code must not
 // pass the symbol itself to a kernel (on the host it names a host-side
-// stand-in); query_scratch_address() looks up the device address instead.
+// stand-in); query_scratch_address() looks up the device address instead,
+// once per device. The cached address belongs to the device's primary
+// context: after cudaDeviceReset it would be stale, and the library does not
+// support a reset within the process.
 namespace {
 static __device__ __align__(256) unsigned char g_query_scratch[MLA_NOALLOC_SCRATCH_BYTES];
 
@@ -373,7 +376,7 @@ int query_scratch_address(void** out) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_query_scratch);
     if (e != cudaSuccess || !p) {
-      set_last_cuda_error(e);
+      set_last_cuda_error(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
       return MLA_ERR_CUDA;
     }
     g_scratch_addr[dev] = p;

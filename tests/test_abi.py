@@ -129,3 +129,64 @@ def test_rope_table_matches_oracle_frequencies(name):
     pos = np.arange(w.rope_table_len)[:, None]
     np.testing.assert_allclose(tab[..., 0], np.cos(pos * inv), rtol=0, atol=2e-7)
     np.testing.assert_allclose(tab[..., 1], np.sin(pos * inv), rtol=0, atol=2e-7)
+
+
+def test_sink_append_takes_at_most_the_fifo_slots():
+    """Frames past the S sinks share W - S frame slots (App. D.4), so one
+    append may carry at most W - S of them: a longer run would write two
+    frames to the same slots. The rule is checked on the host, before any
+    pointer is used (the later residency check then fails on fake pointers,
+    with MLA_ERR_ARG on a GPU machine or MLA_ERR_CUDA without a device)."""
+    lib = V.load()
+    fake = ctypes.c_void_p(1 << 20)
+
+    def append(w, first, n, written):
+        cache = V.mla_cache(c=fake, kr=fake, rope_table=fake, frames_written=written,
+                            cfg=V.make_config(w))
+        return lib.mla_cache_append(ctypes.byref(cache), fake, fake, None, fake, None, first, n,
+                                    None)
+
+    sink = synth.workload("sink")                    # W = 7, S = 1: six FIFO frame slots
+    assert append(sink, 1, 7, 1) == V.MLA_ERR_RANGE  # frames 1..7: seven FIFO frames
+    assert append(sink, 0, 7, 0) != V.MLA_ERR_RANGE  # the sink + six FIFO frames
+    assert append(sink, 1, 6, 1) != V.MLA_ERR_RANGE  # exactly W - S FIFO frames
+    assert append(sink, 955, 6, 958) != V.MLA_ERR_RANGE
+    assert append(sink, 955, 7, 958) == V.MLA_ERR_RANGE
+    w4 = synth.workload("tiny", window_frames=4, sink_frames=1)
+    assert append(w4, 1, 4, 1) == V.MLA_ERR_RANGE    # frames 1 and 4 would share a slot
+    assert append(w4, 1, 3, 1) != V.MLA_ERR_RANGE
+    w2 = synth.workload("tiny", window_frames=4, sink_frames=2)
+    assert append(w2, 1, 3, 1) != V.MLA_ERR_RANGE    # frame 1 is a sink, 2 and 3 fill the FIFO
+    assert append(w2, 1, 4, 1) == V.MLA_ERR_RANGE
+    assert append(w2, 0, 4, 0) != V.MLA_ERR_RANGE
+    plain = synth.workload("tiny")                   # S = 0: the plain ring, n <= W
+    assert append(plain, 0, plain.window_frames, 0) != V.MLA_ERR_RANGE
+
+
+def _aligned_host(nbytes):
+    buf = np.zeros(nbytes + 64, dtype=np.uint8)
+    off = (-buf.ctypes.data) % 64
+    return buf, ctypes.c_void_p(buf.ctypes.data + off)
+
+
+def test_host_memory_is_refused():
+    """Every buffer must be device memory of the current device (the kernels
+    copy tiles with TMA and multicast them within a cluster of this GPU).
+    Host buffers are refused before anything is enqueued: MLA_ERR_ARG where a
+    GPU is present, MLA_ERR_CUDA here without one (no current device)."""
+    lib = V.load()
+    w = synth.workload("tiny")
+    cfg = V.make_config(w)
+    keep, p = [], []
+    for nbytes in (w.slots * w.d_c * 2, w.slots * w.d_r * 2, 1024 * w.d_r * 4,
+                   64 * 12 * w.d_c * 2, 64 * 12 * w.d_r * 2, 64 * 12, 64 * 12 * w.d_c * 2):
+        b, ptr = _aligned_host(nbytes)
+        keep.append(b)
+        p.append(ptr)
+    cache = V.mla_cache(c=p[0], kr=p[1], rope_table=p[2], frames_written=w.window_frames, cfg=cfg)
+    rc = lib.mla_attention_forward(ctypes.byref(cache), p[3], p[4], p[5], 64, p[6], None)
+    assert rc in (V.MLA_ERR_ARG, V.MLA_ERR_CUDA)
+    if rc == V.MLA_ERR_CUDA:
+        assert lib.mla_last_cuda_error() != 0
+    rc = lib.mla_cache_reset(ctypes.byref(cache), None)
+    assert rc in (V.MLA_ERR_ARG, V.MLA_ERR_CUDA)

@@ -28,7 +28,10 @@ def test_reference_arm_prints_one_json_line():
     assert d["steps"] == 2 and d["warmup"] == 0
     assert "workload" in d["config"]
     cb = d["cpu_baseline"]
-    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"]
+    assert cb["kind"] == "oracle" and cb["sample"]
+    # one single-threaded oracle worker per host core
+    assert cb["cores"] == cb["host_cores_available"] == len(os.sched_getaffinity(0))
+    assert "worker processes" in cb["sample"]
     assert cb["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}

@@ -584,3 +584,33 @@ def test_host_argument_errors():
     with pytest.raises(V.MlaError) as e:       # a gap: frame 2 before frames 0, 1
         V.mla_cache_append(cache, x, weights["w_dkv"], None, weights["w_kr"], pos, 2, 1)
     assert e.value.code == V.MLA_ERR_ARG
+
+
+def test_host_and_pinned_memory_refused():
+    """Every buffer must be device memory of the current device: the kernels'
+    TMA copies and cluster multicast address this GPU's own memory only. Host
+    tensors, pageable or pinned, are refused before anything is enqueued."""
+    import ctypes
+    w = small()
+    cfg = V.make_config(w)
+    cache = V.LatentCache(cfg)
+    V.mla_cache_reset(cache)
+    cache.frames_written = w.window_frames
+    q_c, q_r = synth.draw_queries(w, 8, 1)
+    q_pos = synth.grid_positions(w, 0, 1)[:, :8].contiguous()
+    o = torch.empty(1, 8, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    lib = V.load()
+    dev = [q_c.cuda(), q_r.cuda(), q_pos.cuda()]
+    for host in (q_c.clone(), q_c.pin_memory()):
+        args = [host, dev[1], dev[2]]
+        rc = lib.mla_attention_forward(ctypes.byref(cache.struct),
+                                       *[ctypes.c_void_p(t.data_ptr()) for t in args], 8,
+                                       ctypes.c_void_p(o.data_ptr()), None)
+        assert rc == V.MLA_ERR_ARG
+    o_host = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    rc = lib.mla_attention_forward(ctypes.byref(cache.struct),
+                                   *[ctypes.c_void_p(t.data_ptr()) for t in dev], 8,
+                                   ctypes.c_void_p(o_host.data_ptr()), None)
+    assert rc == V.MLA_ERR_ARG
+    V.mla_attention_forward(cache, *dev, o)           # the same call on device memory runs
+    torch.cuda.synchronize()

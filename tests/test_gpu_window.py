@@ -68,10 +68,22 @@ def oracle_window(w, oc, q_c, q_r, q_pos, tokens=None):
 
 
 # ------------------------------------------------------------------ append
+SINK_SCHEDULES = [
+    # mixed chunk sizes, the current chunk rewritten once
+    ([(0, 2), (2, 2), (4, 1), (5, 3), (8, 3), (8, 3), (11, 2)], [0, 10, 11, 12]),
+    # every append as long as the rule allows: the sink and all W - S FIFO
+    # frames at once, then exactly W - S FIFO frames per call
+    ([(0, 4), (4, 3), (7, 3), (7, 3), (10, 3)], [0, 10, 11, 12]),
+]
+
+
+@pytest.mark.parametrize("sched", range(len(SINK_SCHEDULES)))
 @pytest.mark.parametrize("flags", [0, V.MLA_FLAG_SIMT])
-def test_sink_fifo_slots_bit_exact(flags):
+def test_sink_fifo_slots_bit_exact(flags, sched):
     """One-hot projections, no RMSNorm: every stored value is an input value,
-    so the sink + FIFO slot map and the unrotated k^R match bit for bit."""
+    so the sink + FIFO slot map and the unrotated k^R match bit for bit. An
+    append of more than W - S frames past the sinks is refused."""
+    schedule, expect_held = SINK_SCHEDULES[sched]
     w = synth.workload("tiny", grid_h=6, grid_w=7, window_frames=4, sink_frames=1, batch=2)
     cfg = V.make_config(w, flags | V.MLA_FLAG_NO_RMSNORM)
     assert cfg.flags & V.MLA_FLAG_ROTATE_AT_USE
@@ -84,14 +96,19 @@ def test_sink_fifo_slots_bit_exact(flags):
     w_kr[torch.arange(dr), dc + torch.arange(dr)] = 1
     T = w.tokens_per_frame
     frames = {}
-    for i, (first, n) in enumerate([(0, 2), (2, 2), (4, 1), (5, 3), (8, 3), (8, 3), (11, 2)]):
+    for i, (first, n) in enumerate(schedule):
         x = synth.draw_tokens(w, n * T, 800 + i)
         V.mla_cache_append(cache, x.cuda(), w_dkv.cuda(), None, w_kr.cuda(), None, first, n)
         for k in range(n):
             frames[first + k] = x[:, k * T:(k + 1) * T]
     torch.cuda.synchronize()
+    last = cache.frames_written
+    with pytest.raises(V.MlaError) as e:              # frames last-3 .. last: 4 > W - S
+        V.mla_cache_append(cache, synth.draw_tokens(w, 4 * T, 899).cuda(), w_dkv.cuda(), None,
+                           w_kr.cuda(), None, last - 3, 4)
+    assert e.value.code == V.MLA_ERR_RANGE and cache.frames_written == last
     held = O.sink_window_frames(cache.frames_written, w.window_frames, 1)
-    assert held == [0, 10, 11, 12]
+    assert held == expect_held
     c_bits = cache.c.cpu().view(torch.int16)
     k_bits = cache.kr.cpu().view(torch.int16)
     for f in held:
