@@ -362,6 +362,18 @@ int mla_last_cuda_error(void);
  */
 int mla_device_status(int* status, int clear);
 
+/*
+ * Debug builds only (libvideomla_debug.so, built with VMLA_DEBUG_CHECKS=1):
+ * read (and, if clear != 0, reset) the number of query rows whose online
+ * softmax rescaled its running output because the running maximum of the
+ * scores grew by more than 2^8 (in log2 units) from one key block to a later
+ * one (Eq. score; the softmax over the window, Sec. 3.3). Counted by the
+ * tensor-core attention kernels, absorbed and dense, once per (row, block)
+ * that rescales. Synchronises the device. A release build sets *count = 0
+ * and returns MLA_ERR_UNSUPPORTED; MLA_ERR_ARG for a null pointer.
+ */
+int mla_debug_rescale_count(unsigned long long* count, int clear);
+
 /* Library version, e.g. 100 for 0.1.0. */
 int mla_version(void);
 

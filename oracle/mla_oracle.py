@@ -360,7 +360,7 @@ def reference_attention(x_q, pos_q, x_kv, pos_kv, w, head_dim, spec,
     return out[0] if len(out) == 1 else tuple(out)
 
 
-def dense_attention(q, k, v, head_dim):
+def dense_attention(q, k, v, head_dim, return_probs=False):
     """Dense per-head attention, the layout VideoMLA replaces (App. C.1).
 
     q [Nq, H, d_h]; k, v [H, Nk, d_h] (RoPE already applied to q and k).
@@ -370,7 +370,9 @@ def dense_attention(q, k, v, head_dim):
     k = np.asarray(k, dtype=np.float64)
     v = np.asarray(v, dtype=np.float64)
     s = np.einsum("nhd,hjd->nhj", q, k) / math.sqrt(head_dim)
-    return np.einsum("nhj,hjd->nhd", softmax(s, axis=-1), v)
+    p = softmax(s, axis=-1)
+    o = np.einsum("nhj,hjd->nhd", p, v)
+    return (o, p) if return_probs else o
 
 
 # --------------------------------------------------------------------------

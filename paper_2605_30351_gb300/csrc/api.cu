@@ -14,7 +14,15 @@
 namespace vmla {
 namespace {
 
-__device__ int g_device_status = MLA_OK;
+// The device status area every kernel receives as `int* status`: the status
+// word, a pad, then a 64-bit counter that only debug builds advance (rows of
+// the online softmax that rescaled their output; see debug_count_rescale).
+struct alignas(8) DeviceStatusArea {
+  int status;
+  int pad;
+  unsigned long long rescales;
+};
+__device__ DeviceStatusArea g_device_status = {MLA_OK, 0, 0ull};
 
 thread_local int t_last_cuda_error = 0;
 
@@ -625,6 +633,26 @@ const char* mla_status_string(int status) {
 }
 
 int mla_last_cuda_error(void) { return t_last_cuda_error; }
+
+int mla_debug_rescale_count(unsigned long long* count, int clear) {
+  if (!count) return MLA_ERR_ARG;
+#if VMLA_DEBUG_CHECKS
+  int* p = device_status_ptr();
+  if (!p) return MLA_ERR_CUDA;
+  unsigned long long* ctr = reinterpret_cast<unsigned long long*>(p + 2);
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(count, ctr, sizeof(*count), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && clear) {
+    const unsigned long long zero = 0;
+    e = cudaMemcpy(ctr, &zero, sizeof(zero), cudaMemcpyHostToDevice);
+  }
+  return e == cudaSuccess ? MLA_OK : fail_cuda(e);
+#else
+  (void)clear;
+  *count = 0;
+  return MLA_ERR_UNSUPPORTED;
+#endif
+}
 
 int mla_device_status(int* status, int clear) {
   if (!status) return MLA_ERR_ARG;

@@ -262,6 +262,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         alpha = ex2_approx(m_run - m_blk);
         m_run = m_blk;
       }
+      debug_count_rescale(need && row_ok, p.status);
       l_run *= alpha;
       const float neg_m = -m_run;
       // scale-and-shift and the row sum two scores per instruction (paired

@@ -437,6 +437,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         alpha = ex2_approx(m_run - m_blk);
         m_run = m_blk;
       }
+      debug_count_rescale(need && row_ok, p.status);
       l_run *= alpha;
       // P_j in registers before waiting on PV_{j-1}: only the TMEM store
       // below is serialised with the previous PV

@@ -48,6 +48,19 @@ __device__ __forceinline__ bool debug_in_range(long long v, long long lo, long l
   return true;
 }
 
+// Debug builds count the rows of the online softmax that rescale their output
+// (running maximum grown past the lazy-rescale margin) in the 64-bit counter
+// that follows the status word (the status area is {int status; int pad;
+// unsigned long long rescales}); mla_debug_rescale_count reads it. Release
+// builds compile the count away.
+__device__ __forceinline__ void debug_count_rescale(bool rescaled, int* status) {
+#if VMLA_DEBUG_CHECKS
+  if (rescaled && status) atomicAdd(reinterpret_cast<unsigned long long*>(status + 2), 1ull);
+#else
+  (void)rescaled; (void)status;
+#endif
+}
+
 // ----------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)

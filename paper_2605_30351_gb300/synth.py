@@ -21,7 +21,8 @@ import numpy as np
 import torch
 
 __all__ = ["Workload", "WORKLOADS", "workload", "bf16", "draw_layer_weights",
-           "draw_tokens", "grid_positions", "frame_coords", "draw_queries", "draw_cache_rows"]
+           "draw_tokens", "grid_positions", "frame_coords", "draw_queries", "draw_cache_rows",
+           "unit_vectors", "fill_normal_"]
 
 
 @dataclass(frozen=True)
@@ -148,19 +149,45 @@ def frame_coords(w):
     return torch.from_numpy(np.stack([hh, ww], axis=-1).astype(np.int32))
 
 
-def draw_queries(w, n_tokens, seed, batch=None):
-    """Absorbed content queries q_c [B, n, H, d_c] and unrotated q_r [B, n, H, d_r]."""
+def draw_queries(w, n_tokens, seed, batch=None, qc_std=None, qr_std=1.0, as_float64=False):
+    """Absorbed content queries q_c [B, n, H, d_c] and unrotated q_r [B, n, H, d_r].
+
+    q_c ~ N(0, qc_std^2) with qc_std = sqrt(d_nope / d_c) by default; q_r ~
+    N(0, qr_std^2). as_float64 returns the float64 draws before rounding (for
+    callers that build structured inputs and round them once themselves)."""
     rng = np.random.default_rng(seed)
     B = w.batch if batch is None else batch
     dn = w.head_dim - w.d_r
-    q_c = _normal(rng, (B, n_tokens, w.heads, w.d_c), (dn / w.d_c) ** 0.5)
-    q_r = _normal(rng, (B, n_tokens, w.heads, w.d_r), 1.0)
+    q_c = _normal(rng, (B, n_tokens, w.heads, w.d_c),
+                  (dn / w.d_c) ** 0.5 if qc_std is None else qc_std)
+    q_r = _normal(rng, (B, n_tokens, w.heads, w.d_r), qr_std)
+    if as_float64:
+        return q_c, q_r
     return bf16(q_c), bf16(q_r)
 
 
-def draw_cache_rows(w, n_rows, seed, batch=None):
+def unit_vectors(n, d, seed):
+    """n random directions in R^d (rows of unit length), float64."""
+    rng = np.random.default_rng(seed)
+    u = rng.standard_normal((n, d))
+    return u / np.linalg.norm(u, axis=1, keepdims=True)
+
+
+def draw_cache_rows(w, n_rows, seed, batch=None, as_float64=False):
     """Cache contents c [B, n, d_c] ~ N(0,1) and rotated keys k [B, n, d_r] ~ N(0,1)."""
     rng = np.random.default_rng(seed)
     B = w.batch if batch is None else batch
-    return (bf16(rng.standard_normal((B, n_rows, w.d_c))),
-            bf16(rng.standard_normal((B, n_rows, w.d_r))))
+    c, k = rng.standard_normal((B, n_rows, w.d_c)), rng.standard_normal((B, n_rows, w.d_r))
+    if as_float64:
+        return c, k
+    return bf16(c), bf16(k)
+
+
+def fill_normal_(t, seed, std=1.0):
+    """Fill a (CUDA) tensor in place with N(0, std^2) draws of a seeded torch
+    generator on its device, rounded once to the tensor's dtype: inputs of
+    batches too large to draw on the host (both sides read the same values
+    back)."""
+    g = torch.Generator(device=t.device).manual_seed(seed)
+    t.normal_(0.0, std, generator=g)
+    return t

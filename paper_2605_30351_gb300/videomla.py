@@ -34,7 +34,8 @@ EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
            "mla_query_prologue_noalloc", "mla_output_projection", "mla_dense_attention_forward",
            "mla_window_workspace_bytes", "mla_attention_window_forward", "mla_decompress_window",
-           "mla_selftest_bounded_wait", "mla_status_string", "mla_last_cuda_error", "mla_device_status", "mla_version")
+           "mla_selftest_bounded_wait", "mla_status_string", "mla_last_cuda_error", "mla_device_status",
+           "mla_debug_rescale_count", "mla_version")
 
 
 class mla_config(ctypes.Structure):
@@ -90,6 +91,7 @@ def load():
     lib.mla_status_string.restype = ctypes.c_char_p
     lib.mla_last_cuda_error.argtypes = []
     lib.mla_device_status.argtypes = [P(I), I]
+    lib.mla_debug_rescale_count.argtypes = [P(ctypes.c_ulonglong), I]
     lib.mla_version.argtypes = []
     lib.mla_absorb_weights.argtypes = [P(mla_config), VP, VP, VP, VP, VP, VP, VP, VP, VP]
     lib.mla_query_workspace_bytes.argtypes = [P(mla_config), I]
@@ -110,7 +112,8 @@ def load():
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
                  "mla_query_prologue_noalloc", "mla_output_projection",
                  "mla_dense_attention_forward", "mla_attention_window_forward",
-                 "mla_decompress_window", "mla_selftest_bounded_wait"):
+                 "mla_decompress_window", "mla_selftest_bounded_wait",
+                 "mla_debug_rescale_count"):
         getattr(lib, name).restype = I
     _lib = lib
     return lib
@@ -374,3 +377,12 @@ def mla_device_status(clear=True):
     st = ctypes.c_int(0)
     _check("mla_device_status", load().mla_device_status(ctypes.byref(st), int(bool(clear))))
     return st.value
+
+
+def mla_debug_rescale_count(clear=True):
+    """Rows whose online softmax rescaled its output (debug build only; a
+    release build raises MlaError with MLA_ERR_UNSUPPORTED)."""
+    n = ctypes.c_ulonglong(0)
+    _check("mla_debug_rescale_count",
+           load().mla_debug_rescale_count(ctypes.byref(n), int(bool(clear))))
+    return n.value

@@ -2,8 +2,11 @@
 named on the command line (release or debug build), runs a fixed set of
 calls (append + attention on the 21-frame ring, the sink window, the
 decompression, the query prologue and output projection; the append's
-cluster and split forms and the split-output attention at d_c = 256 and 512)
-on seeded inputs and saves every output plus the device status word."""
+cluster and split forms and the split-output attention at d_c = 256 and 512;
+the online softmax's rescale branch in the absorbed and dense kernels) on
+seeded inputs and saves every output, the device status word and the debug
+build's count of softmax rescales (-1 for the release build, which does not
+count)."""
 
 import os
 import sys
@@ -12,6 +15,7 @@ import torch
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 sys.path.insert(0, ROOT)
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
 
 from paper_2605_30351_gb300 import synth  # noqa: E402
 from paper_2605_30351_gb300 import videomla as V  # noqa: E402
@@ -79,6 +83,34 @@ def main(lib_path, out_path):
                                 o)
         torch.cuda.synchronize()
         out[f"c_{d_c}"], out[f"kr_{d_c}"], out[f"o_{d_c}"] = cache.c.cpu(), cache.kr.cpu(), o.cpu()
+    # the online softmax's rescale branch: a dominant key in the last key
+    # block for a third of the rows, absorbed (390 keys) and dense (500 keys)
+    from test_gpu_softmax import absorbed_inputs, dense_inputs
+    try:
+        V.mla_debug_rescale_count(clear=True)
+    except V.MlaError as e:
+        assert e.code == V.MLA_ERR_UNSUPPORTED  # the release build does not count
+    w = synth.workload("tiny", grid_h=10, grid_w=13, window_frames=3, batch=2,
+                       rope_pairs=(6, 5, 5))
+    q_c, q_r, c, k, _ = absorbed_inputs(w, 40, "late", 90)
+    cache = V.LatentCache(V.make_config(w))
+    cache.c.copy_(c)
+    cache.kr.copy_(k)
+    cache.frames_written = w.window_frames
+    o = torch.empty(w.batch, 40, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    V.mla_attention_forward(cache, q_c.cuda(), q_r.cuda(),
+                            synth.grid_positions(w, 2, 1)[:, :40].contiguous().cuda(), o)
+    wd = synth.workload("tiny", batch=2)
+    q, kd, vd, _ = dense_inputs(wd, 300, 500, "late", 91)
+    od = torch.empty(q.shape, dtype=torch.bfloat16, device="cuda")
+    V.mla_dense_attention_forward(V.make_config(wd), q.cuda(), kd.cuda(), vd.cuda(), 500, od)
+    torch.cuda.synchronize()
+    out["o_late"], out["o_dense_late"] = o.cpu(), od.cpu()
+    try:
+        out["rescales"] = V.mla_debug_rescale_count(clear=True)
+    except V.MlaError as e:
+        assert e.code == V.MLA_ERR_UNSUPPORTED
+        out["rescales"] = -1
     out["status"] = V.mla_device_status(clear=True)
     torch.save(out, out_path)
 

@@ -1,6 +1,8 @@
 """The debug build (device-side index checks on, -DVMLA_DEBUG_CHECKS=1): it
-compiles, raises no false alarm on valid inputs, and computes bit-for-bit
-what the release build computes. Each build runs in a process of its own."""
+compiles, raises no false alarm on valid inputs, computes bit-for-bit what the
+release build computes, and counts the online softmax's output rescales,
+which inputs with a dominant key in the last key block must trigger. Each
+build runs in a process of its own."""
 
 import os
 import subprocess
@@ -29,6 +31,11 @@ def test_debug_build_matches_release_without_false_alarms(tmp_path):
         assert r.returncode == 0, r.stderr[-3000:]
         outs[name] = torch.load(path)
     assert outs["debug"]["status"] == 0 and outs["release"]["status"] == 0
+    # the planted late key makes a third of the rows rescale their output at
+    # the last key block: 2 x 160 absorbed rows and 2 x 100 x 12 dense rows
+    # (at least; earlier blocks may rescale some rows too)
+    assert outs["release"]["rescales"] == -1
+    assert outs["debug"]["rescales"] >= 2 * 160 + 2 * 100 * 12, outs["debug"]["rescales"]
     for key, t in outs["release"].items():
-        if key != "status":
+        if key not in ("status", "rescales"):
             assert torch.equal(t, outs["debug"][key]), key

@@ -29,6 +29,24 @@ def assert_close(got, ref, max_abs=MAX_ABS, rel_l2=REL_L2, what=""):
     return ma, rl
 
 
+def assert_rows_close(got, ref, what, row_rel=1e-2):
+    """Per row (last axis = one output row): rel-L2 <= row_rel and max-abs <=
+    row_rel * max|ref row|; over all rows the bounds of assert_close."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    got = got.reshape(-1, got.shape[-1])
+    ref = ref.reshape(-1, ref.shape[-1])
+    assert_close(got, ref, what=what)
+    d = got - ref
+    rel = np.linalg.norm(d, axis=1) / np.maximum(np.linalg.norm(ref, axis=1), 1e-30)
+    mab = np.max(np.abs(d), axis=1) / np.maximum(np.max(np.abs(ref), axis=1), 1e-30)
+    worst = int(np.argmax(rel))
+    assert rel.max() <= row_rel, f"{what}: row {worst} rel-L2 {rel[worst]:.3e}"
+    worst = int(np.argmax(mab))
+    assert mab.max() <= row_rel, f"{what}: row {worst} max-abs/max|ref| {mab[worst]:.3e}"
+
+
 def f64(t):
     return t.detach().float().cpu().numpy().astype(np.float64)
 
