@@ -70,3 +70,50 @@ def test_noalloc_refuses_requests_beyond_its_scratch(layer):
                                              w.chunk_tokens, fake, fake, None)
     assert rc == V.MLA_ERR_TOO_LARGE
     assert "no-allocation" in V.load().mla_status_string(rc).decode()
+
+
+def _compare_twice(w, cfg, wt, w_qcat, nq, seeds):
+    ws = torch.empty(V.mla_query_workspace_bytes(cfg, nq), dtype=torch.uint8, device="cuda")
+    for call, seed in enumerate(seeds):
+        x = synth.draw_tokens(w, nq, seed).cuda()
+        ref_c, ref_r = _outputs(w, nq)
+        V.mla_query_prologue(cfg, x, wt["w_dq"], w_qcat, ws, ref_c, ref_r)
+        got_c, got_r = _outputs(w, nq)
+        V.mla_query_prologue_noalloc(cfg, x, wt["w_dq"], w_qcat, got_c, got_r)
+        torch.cuda.synchronize()
+        assert_close(f64(got_c), f64(ref_c), what=f"q_c, call {call}")
+        assert_close(f64(got_r), f64(ref_r), what=f"q_r, call {call}")
+    assert V.mla_device_status(clear=True) == V.MLA_OK
+
+
+def test_noalloc_wide_tiles_match_workspace_entry_point():
+    """A query latent of d_q = 128 over five Wan chunks (23,400 rows: 183 row
+    tiles) takes the 256-wide first GEMM, whose partial sums of squares use a
+    different tile count in the scratch; 6.1 MB still fits the fixed array."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    w = synth.workload("wan", d_q=128, batch=5)
+    cfg = V.make_config(w)
+    nq = w.chunk_tokens
+    need = V.mla_query_workspace_bytes(cfg, nq)
+    assert need <= V.MLA_NOALLOC_SCRATCH_BYTES and (w.batch * nq + 127) // 128 >= 152
+    wt = {k: v.cuda() for k, v in synth.draw_layer_weights(w, seed=311).items()}
+    w_qcat, _ = V.mla_absorb_weights(cfg, wt["w_uq"], wt["w_uk"], wt["w_qr"], wt["gamma_q"],
+                                     wt["w_uv"], wt["w_o"])
+    _compare_twice(w, cfg, wt, w_qcat, nq, (312, 313))
+
+
+def test_noalloc_at_the_scratch_limit(layer):
+    """The largest query count whose intermediate buffer fits the fixed array
+    exactly (d_q = 768: 1552 bytes per token) is accepted and correct; one
+    token more is refused before anything is queued."""
+    w, cfg, wt, w_qcat = layer
+    nq = V.MLA_NOALLOC_SCRATCH_BYTES // 1552
+    assert V.mla_query_workspace_bytes(cfg, nq) <= V.MLA_NOALLOC_SCRATCH_BYTES
+    assert V.mla_query_workspace_bytes(cfg, nq + 1) > V.MLA_NOALLOC_SCRATCH_BYTES
+    _compare_twice(w, cfg, wt, w_qcat, nq, (314, 315))
+    x = synth.draw_tokens(w, nq + 1, 316).cuda()
+    got_c, got_r = _outputs(w, nq + 1)
+    with pytest.raises(V.MlaError) as e:
+        V.mla_query_prologue_noalloc(cfg, x, wt["w_dq"], w_qcat, got_c, got_r)
+    assert e.value.code == V.MLA_ERR_TOO_LARGE
