@@ -361,10 +361,6 @@ def run_ours(args, w):
     # one set per layer of a step, or N_SETS rotating sets for a one-layer step
     n_sets = max(w.layers, N_SETS)
     sets = [LayerSet(w, 1000 + 17 * i, V) for i in range(n_sets)]
-    # one attention workspace for every layer (the calls run in stream order):
-    # the last, partial wave of row tiles is split over the SMs by key range
-    ws_attn = torch.empty(V.mla_attention_workspace_bytes(sets[0].cache.cfg, w.chunk_tokens),
-                          dtype=torch.uint8, device="cuda")
     attn_l, app_l = flops_per_layer(w)
     attn_fl, app_fl = attn_l * w.layers, app_l * w.layers
 
@@ -378,7 +374,7 @@ def run_ours(args, w):
         if s.window:
             V.mla_attention_window_forward(s.cache, s.q_c, s.q_r, s.pos, s.hw, s.ws, s.o, stream)
         else:
-            V.mla_attention_forward_ws(s.cache, s.q_c, s.q_r, s.pos, ws_attn, s.o, stream)
+            V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
         if ev is not None:
             ev[2].record(stream)
 
@@ -537,8 +533,7 @@ def run_ours(args, w):
             "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
             "peak_source": f"{peaks['source']} bf16 dense ({peak_kind}: {peak_why})",
             "kernel": ("window_assemble_kernel + mla_attn_tc_kernel<192,32,2,128> (events around both)"
-                       if w.sink_frames else "mla_attn_tc_kernel<192,32,2,128> (last wave split "
-                       "by key range: mla_attention_forward_ws, plus its counter memset)"),
+                       if w.sink_frames else "mla_attn_tc_kernel<192,32,2,128>"),
             "algorithmic_flops_per_launch": attn_l,
             "traffic": (profiled_traffic("attn_tc_wan_traffic.json", "attn_tc.cu")
                         if w.batch == 1 else None),
@@ -833,8 +828,6 @@ def run_layer(args, w):
         s.w_qcat, s.w_b = V.mla_absorb_weights(cfg, wt["w_uq"], wt["w_uk"], wt["w_qr"],
                                                wt["gamma_q"], wt["w_uv"], wt["w_o"])
         s.ws_q = torch.empty(V.mla_query_workspace_bytes(cfg, nq), dtype=torch.uint8, device="cuda")
-        s.ws_a = torch.empty(V.mla_attention_workspace_bytes(cfg, nq), dtype=torch.uint8,
-                             device="cuda")
         s.y = torch.empty(w.batch, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
         sets.append(s)
 
@@ -852,7 +845,7 @@ def run_layer(args, w):
         if s.window:
             V.mla_attention_window_forward(s.cache, s.q_c, s.q_r, s.pos, s.hw, s.ws, s.o, stream)
         else:
-            V.mla_attention_forward_ws(s.cache, s.q_c, s.q_r, s.pos, s.ws_a, s.o, stream)
+            V.mla_attention_forward(s.cache, s.q_c, s.q_r, s.pos, s.o, stream)
         if ev is not None:
             ev[3].record(stream)
         V.mla_output_projection(cfg, s.o, s.w_b, s.y, stream)

@@ -198,35 +198,6 @@ int mla_attention_forward(const mla_cache* cache, const void* q_c,
                           const void* q_r, const int* q_pos, int Nq,
                           void* o_lat, void* stream);
 
-/* Bytes of caller-owned device workspace mla_attention_forward_ws needs on
- * the CURRENT device (it depends on the device's SM count and on d_c, not on
- * Nq); 0 on a bad config, Nq < 1, or without a current device. */
-unsigned long long mla_attention_workspace_bytes(const mla_config* cfg, int Nq);
-
-/*
- * mla_attention_forward with a caller workspace, the same computation
- * (Eq. score; App. E) and the same arguments, plus:
- *  workspace  device memory of at least mla_attention_workspace_bytes(cfg,
- *             Nq) bytes on the current device, 16-byte aligned, owned by the
- *             caller; scratch for this call only (each call zeroes what it
- *             needs; calls that overlap on the GPU must not share it)
- * With it, the last wave of 128-row tiles no longer leaves SMs idle: the
- * row tiles that do not fill a whole wave have their key blocks shared out
- * evenly over every SM pair of that wave, each pair taking a contiguous key
- * range of at most two tiles. A piece writes its unnormalised latent output
- * and its softmax running maximum and sum (fp32) to the workspace, and the
- * last piece of a tile to finish combines them: o = sum_k 2^(m_k - m) O_k /
- * sum_k 2^(m_k - m) l_k, m = max_k m_k (the same online softmax, split over
- * keys). The split runs only for d_c <= 192 with at least one full wave of
- * tile pairs before the partial one; otherwise this call is
- * mla_attention_forward. Each such call enqueues a small memset of the
- * workspace's counters before the kernel. MLA_ERR_ARG for a workspace that
- * is too small, in addition to mla_attention_forward's errors.
- */
-int mla_attention_forward_ws(const mla_cache* cache, const void* q_c, const void* q_r,
-                             const int* q_pos, int Nq, void* workspace,
-                             unsigned long long workspace_bytes, void* o_lat, void* stream);
-
 /* Bytes of caller-owned device workspace mla_attention_window_forward needs
  * for Nq query tokens per batch element (0 on a bad config). */
 unsigned long long mla_window_workspace_bytes(const mla_config* cfg, int Nq);

@@ -145,8 +145,7 @@ bool rotate_at_use(const mla_config& c) { return (c.flags & MLA_FLAG_ROTATE_AT_U
 // Absorbed-form attention over the valid slots, with the given positional
 // keys and query positions.
 int run_attention(const mla_cache* cache, const void* q_c, const void* q_r, const int* q_pos,
-                  int Nq, const void* kr, void* o_lat, cudaStream_t stream,
-                  void* split_ws = nullptr, unsigned long long split_ws_bytes = 0) {
+                  int Nq, const void* kr, void* o_lat, cudaStream_t stream) {
   const mla_config& c = cache->cfg;
   const long long n_valid = valid_slots(*cache);
   if (n_valid < 1) return MLA_ERR_ARG;
@@ -173,8 +172,6 @@ int run_attention(const mla_cache* cache, const void* q_c, const void* q_r, cons
   a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(c.head_dim)));
   a.status = device_status_ptr();
   a.stream = stream;
-  a.split_ws = split_ws;
-  a.split_ws_bytes = split_ws_bytes;
   if (!a.status) return MLA_ERR_CUDA;
   return (c.flags & MLA_FLAG_SIMT) ? launch_attention_simt(a) : launch_attention_tc(a);
 }
@@ -360,41 +357,6 @@ int mla_attention_forward(const mla_cache* cache, const void* q_c, const void* q
   if (rc != MLA_OK) return rc;
   return run_attention(cache, q_c, q_r, q_pos, Nq, cache->kr, o_lat,
                        static_cast<cudaStream_t>(stream));
-}
-
-unsigned long long mla_attention_workspace_bytes(const mla_config* cfg, int Nq) {
-  if (check_config(cfg) != MLA_OK || Nq < 1) return 0;
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
-    (void)cudaGetLastError();
-    return 0;
-  }
-  return attention_split_workspace_bytes(cfg->d_c, sms);
-}
-
-int mla_attention_forward_ws(const mla_cache* cache, const void* q_c, const void* q_r,
-                             const int* q_pos, int Nq, void* workspace,
-                             unsigned long long workspace_bytes, void* o_lat, void* stream) {
-  if (!cache) return MLA_ERR_ARG;
-  int rc = check_config(&cache->cfg);
-  if (rc != MLA_OK) return rc;
-  const mla_config& c = cache->cfg;
-  if (!cache->c || !cache->kr || !cache->rope_table || !q_c || !q_r || !q_pos || !o_lat ||
-      !workspace)
-    return MLA_ERR_ARG;
-  if (!aligned16(cache->c) || !aligned16(cache->kr) || !aligned16(q_c) || !aligned16(q_r) ||
-      !aligned16(o_lat) || !aligned16(cache->rope_table) || !aligned16(workspace) ||
-      (reinterpret_cast<uintptr_t>(q_pos) & 3u))
-    return MLA_ERR_ARG;
-  if (Nq < 1 || rotate_at_use(c)) return MLA_ERR_ARG;
-  const unsigned long long need = mla_attention_workspace_bytes(&c, Nq);
-  if (need == 0) return fail_cuda(cudaErrorNoDevice);
-  if (workspace_bytes < need) return MLA_ERR_ARG;
-  rc = check_resident({cache->c, cache->kr, cache->rope_table, q_c, q_r, q_pos, o_lat, workspace});
-  if (rc != MLA_OK) return rc;
-  return run_attention(cache, q_c, q_r, q_pos, Nq, cache->kr, o_lat,
-                       static_cast<cudaStream_t>(stream), workspace, workspace_bytes);
 }
 
 int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* w_uv, void* k,

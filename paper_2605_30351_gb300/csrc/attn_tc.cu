@@ -112,34 +112,7 @@ struct AttnKParams {
   int rows, heads, n_valid, rope_len, pairs_t, pairs_h;
   float scale_log2;
   int* status;
-  // Work split. Work unit = one cluster's row tile(s) ("pair tile"); the
-  // pair tiles of all batch elements are numbered g = b * pt_per_b + pt.
-  // Clusters g < dp_pairs take pair tile g over the whole window. The
-  // clusters after them ("stream-K slots", sk_slots of them) share the keys
-  // of the remaining pair tiles: slot s takes the flat key-block units
-  // [s * sk_units / sk_slots, (s + 1) * sk_units / sk_slots) of those tiles
-  // (unit = (pair tile, key block)), at most two tiles' pieces. A piece
-  // that is not a whole tile writes its unnormalised output and its softmax
-  // statistics to the workspace; the last piece of a tile to finish
-  // combines them.
-  int pt_per_b, dp_pairs, sk_slots;
-  long long sk_units;
-  float4* sk_part;      // [slot][piece][cta][d_v / 4][128] unnormalised output
-  float* sk_ml;         // [slot][piece][cta][2][128] running max (log2) and sum
-  int* sk_count;        // [stream-K pair tile][cta] pieces finished (zeroed per call)
 };
-
-// A contiguous key range [jb, je) of one row tile (or CTA pair's tiles).
-struct AttnPiece {
-  int b, pt, jb, je;
-  int sk_tile;  // stream-K pair tile index (g - dp_pairs), or -1: the whole window
-  int part;     // which piece of its slot (0 or 1)
-};
-
-// Slot of flat unit u: the largest s with floor(s * U / S) <= u.
-__device__ __forceinline__ int sk_slot_of(long long u, long long units, int slots) {
-  return static_cast<int>(((u + 1) * slots - 1) / units);
-}
 
 template <int DC, int DR, int CL, int BN, int DV>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -167,48 +140,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* p_full = s_free + 1;
   uint64_t* pv_done = p_full + 1;
   uint64_t* mma_drain = pv_done + 1;  // [2]: one per issuing thread
-  uint64_t* sk_done = mma_drain + 2;  // a stream-K piece's partial is in the workspace
-  uint64_t* sk_go = sk_done + 1;      // ... and last_flag says whether to combine
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sk_go + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_drain + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  volatile int* last_flag = abort_flag + 1;  // this CTA finished a tile's last piece
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-  const int vpart = S::kSplit > 1 ? crank : 0;  // which DV output columns
+  const int b = blockIdx.y;
+  const int tile = blockIdx.x / S::kSplit;
+  const int vpart = blockIdx.x - tile * S::kSplit;  // which DV output columns
+  const int row0 = tile * kBM;
   const int nblk = (p.n_valid + kBN - 1) / kBN;
   const WaitCtx wc{abort_flag, p.status};
-
-  // this cluster's pieces: one whole pair tile, or up to two stream-K pieces
-  AttnPiece pc[2];
-  int npc = 1;
-  const int g = blockIdx.y * static_cast<int>(gridDim.x / CL) + static_cast<int>(blockIdx.x / CL);
-  {
-    if (g < p.dp_pairs || !S::kQinTmem) {
-      pc[0] = {g / p.pt_per_b, g % p.pt_per_b, 0, nblk, -1, 0};
-    } else {
-      const long long s = g - p.dp_pairs;
-      long long u = s * p.sk_units / p.sk_slots;
-      const long long u1 = (s + 1) * p.sk_units / p.sk_slots;
-      npc = 0;
-      while (u < u1 && npc < 2) {
-        const int q = static_cast<int>(u / nblk);
-        const int jb = static_cast<int>(u - static_cast<long long>(q) * nblk);
-        const int je = static_cast<int>(min(static_cast<long long>(nblk), jb + (u1 - u)));
-        const int gq = p.dp_pairs + q;
-        const bool whole = jb == 0 && je == nblk;
-        pc[npc] = {gq / p.pt_per_b, gq % p.pt_per_b, jb, je, whole ? -1 : q, npc};
-        u += je - jb;
-        ++npc;
-      }
-      // a slot spans less than one tile's keys, so at most two pieces
-      if (u < u1 && threadIdx.x == 0) record_status(p.status, MLA_ERR_UNSUPPORTED);
-    }
-  }
-  auto piece_row0 = [&](const AttnPiece& c) {
-    return (S::kSplit > 1 ? c.pt : c.pt * CL + crank) * kBM;
-  };
 
   if (threadIdx.x == 0) {
     mbar_init(q_tma_full, 1);
@@ -223,8 +165,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(pv_done, 1);
     mbar_init(&mma_drain[0], 1);
     mbar_init(&mma_drain[1], 1);
-    mbar_init(sk_done, kBM);
-    mbar_init(sk_go, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -238,8 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   // the peer's barriers must be initialised before any multicast lands
   if constexpr (CL > 1) cluster_sync();
-  int total_blocks = 0;
-  for (int k = 0; k < npc; ++k) total_blocks += pc[k].je - pc[k].jb;
+  const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -250,41 +189,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_prefetch_desc(&tm_qc);
         mbar_arrive_expect_tx(q_tma_full, S::kQcSmem * kBM * 2);
         for (int cb = 0; cb < S::kQcSmem / 64; ++cb)
-          tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, S::kQcTmem + cb * 64,
-                      piece_row0(pc[0]), pc[0].b);
+          tma_load_3d(sQ + cb * 16384, &tm_qc, q_tma_full, S::kQcTmem + cb * 64, row0, b);
       }
       int issued = 0;
-      bool ok = true;
-      for (int k = 0, t = 0; ok && k < npc; ++k) {
-        const int b = pc[k].b;
-        for (int j = pc[k].jb; j < pc[k].je; ++j, ++t) {
-          const int st = t % NST;
-          if (t >= NST && !mbar_wait(&kv_empty[st], ((t / NST) - 1) & 1, wc)) {
-            ok = false;
-            break;
+      for (int j = 0; j < nblk; ++j) {
+        const int st = j % NST;
+        if (j >= NST && !mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, wc)) break;
+        uint8_t* kv = sKV + st * S::kTileBytes;
+        mbar_arrive_expect_tx(&kv_full[st], S::kTileBytes);
+        if constexpr (CL == 1) {
+          for (int cb = 0; cb < DC / 64; ++cb)
+            tma_load_3d(kv + cb * S::kCBox, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
+          tma_load_3d(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b);
+        } else {
+          // each CTA fetches every other box once and multicasts it to both
+          for (int bx = crank; bx <= DC / 64; bx += CL) {
+            if (bx < DC / 64)
+              tma_load_3d_mc(kv + bx * S::kCBox, &tm_c, &kv_full[st], bx * 64, j * kBN, b, kPair);
+            else
+              tma_load_3d_mc(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b, kPair);
           }
-          uint8_t* kv = sKV + st * S::kTileBytes;
-          mbar_arrive_expect_tx(&kv_full[st], S::kTileBytes);
-          if constexpr (CL == 1) {
-            for (int cb = 0; cb < DC / 64; ++cb)
-              tma_load_3d(kv + cb * S::kCBox, &tm_c, &kv_full[st], cb * 64, j * kBN, b);
-            tma_load_3d(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b);
-          } else {
-            // each CTA fetches every other box once and multicasts it to both
-            for (int bx = crank; bx <= DC / 64; bx += CL) {
-              if (bx < DC / 64)
-                tma_load_3d_mc(kv + bx * S::kCBox, &tm_c, &kv_full[st], bx * 64, j * kBN, b,
-                               kPair);
-              else
-                tma_load_3d_mc(kv + S::kKrOff, &tm_kr, &kv_full[st], 0, j * kBN, b, kPair);
-            }
-          }
-          issued = t + 1;
         }
+        issued = j + 1;
       }
       // every stage's last use must be released before the CTA may exit
-      for (int st = 0; st < NST && st < total_blocks && !*abort_flag; ++st)
-        mbar_wait(&kv_empty[st], (((total_blocks - st + NST - 1) / NST) - 1) & 1, wc);
+      for (int st = 0; st < NST && st < nblk && !*abort_flag; ++st)
+        mbar_wait(&kv_empty[st], (((nblk - st + NST - 1) / NST) - 1) & 1, wc);
       if (*abort_flag) {  // let every copy this CTA started land before exit
         if constexpr (!S::kQinTmem) mbar_wait_drain(q_tma_full, 0, p.status);
         for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
@@ -295,54 +225,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------ QK^T issuer
     if (lane == 0) {
-      bool ok = true;
-      if constexpr (!S::kQinTmem) ok = mbar_wait(q_tma_full, 0, wc);
+      bool ok = mbar_wait(q_ready, 0, wc);
+      if constexpr (!S::kQinTmem) ok = ok && mbar_wait(q_tma_full, 0, wc);
+      tc_fence_after();
       const uint32_t qa = smem_u32(sQ);
-      for (int k = 0, t = 0; ok && k < npc; ++k) {
-        // Q of this piece's rows is in place (TMEM, and shared memory for q_r)
-        if (!mbar_wait(q_ready, k & 1, wc)) {
+      for (int j = 0; ok && j < nblk; ++j) {
+        // S = Q K_j^T; S's previous contents (block j-1) must have been read
+        if (j >= 1 && !mbar_wait(s_free, (j - 1) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        const int st = j % NST;
+        if (!mbar_wait(&kv_full[st], (j / NST) & 1, wc)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        for (int j = pc[k].jb; j < pc[k].je; ++j, ++t) {
-          // S = Q K_j^T; S's previous contents (block t-1) must have been read
-          if (t >= 1 && !mbar_wait(s_free, (t - 1) & 1, wc)) {
-            ok = false;
-            break;
-          }
-          const int st = t % NST;
-          if (!mbar_wait(&kv_full[st], (t / NST) & 1, wc)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t ka = smem_u32(sKV) + st * S::kTileBytes;
+        const uint32_t ka = smem_u32(sKV) + st * S::kTileBytes;
 #pragma unroll
-          for (int cb = 0; cb < DC / 64; ++cb)
+        for (int cb = 0; cb < DC / 64; ++cb)
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t bd = sdesc(ka + cb * S::kCBox + kk * 32, 16, 1024, kSw128);
-              const uint32_t acc = (cb | kk) != 0 ? 1u : 0u;
-              if (cb < S::kQcTmem / 64)  // resolved at compile time (unrolled)
-                umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + (cb * 4 + kk) * 8, bd, S::kIdescQK,
-                        acc);
-              else
-                umma_ss(tmem + S::kTmemS,
-                        sdesc(qa + (cb - S::kQcTmem / 64) * 16384 + kk * 32, 16, 1024, kSw128),
-                        bd, S::kIdescQK, acc);
-            }
-#pragma unroll
-          for (int kk = 0; kk < DR / 16; ++kk) {
-            const uint64_t bd = sdesc(ka + S::kKrOff + kk * 32, 16, S::kKrSbo, S::kKrSw);
-            if constexpr (S::kQinTmem)
-              umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + DC / 2 + kk * 8, bd, S::kIdescQK, 1u);
+          for (int k = 0; k < 4; ++k) {
+            const uint64_t bd = sdesc(ka + cb * S::kCBox + k * 32, 16, 1024, kSw128);
+            const uint32_t acc = (cb | k) != 0 ? 1u : 0u;
+            if (cb < S::kQcTmem / 64)  // resolved at compile time (unrolled)
+              umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + (cb * 4 + k) * 8, bd, S::kIdescQK, acc);
             else
-              umma_ss(tmem + S::kTmemS, sdesc(qa + S::kQKrOff + kk * 32, 16, S::kKrSbo, S::kKrSw),
-                      bd, S::kIdescQK, 1u);
+              umma_ss(tmem + S::kTmemS,
+                      sdesc(qa + (cb - S::kQcTmem / 64) * 16384 + k * 32, 16, 1024, kSw128), bd,
+                      S::kIdescQK, acc);
           }
-          umma_commit(s_full);
+#pragma unroll
+        for (int k = 0; k < DR / 16; ++k) {
+          const uint64_t bd = sdesc(ka + S::kKrOff + k * 32, 16, S::kKrSbo, S::kKrSw);
+          if constexpr (S::kQinTmem)
+            umma_ts(tmem + S::kTmemS, tmem + S::kTmemQ + DC / 2 + k * 8, bd, S::kIdescQK, 1u);
+          else
+            umma_ss(tmem + S::kTmemS, sdesc(qa + S::kQKrOff + k * 32, 16, S::kKrSbo, S::kKrSw),
+                    bd, S::kIdescQK, 1u);
         }
+        umma_commit(s_full);
       }
       if (!ok) {  // wait for every MMA this thread issued before TMEM is freed
         umma_commit(&mma_drain[0]);
@@ -354,28 +276,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     // --------------------------------------------------------- PV issuer
     if (lane == 0) {
       bool ok = true;
-      for (int k = 0, t = 0; ok && k < npc; ++k) {
-        for (int j = pc[k].jb; j < pc[k].je; ++j, ++t) {
-          // O += P_t V_t, V = this CTA's DV of the first d_c columns of block
-          // t's stage (MN-major); a piece's first block starts O afresh
-          if (!mbar_wait(p_full, t & 1, wc)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const int st = t % NST;
-          const uint32_t va = smem_u32(sKV) + st * S::kTileBytes + vpart * (DV / 64) * S::kCBox;
-#pragma unroll
-          for (int ss = 0; ss < kBN / 16; ++ss)
-            umma_ts(tmem + S::kTmemO, tmem + S::kTmemP + ss * 8,
-                    sdesc(va + ss * 2048, S::kCBox, 1024, kSw128), S::kIdescPV,
-                    (j > pc[k].jb || ss > 0) ? 1u : 0u);
-          if constexpr (CL == 1)
-            umma_commit(&kv_empty[st]);
-          else
-            umma_commit_mc(&kv_empty[st], kPair);
-          umma_commit(pv_done);
+      for (int i = 0; ok && i < nblk; ++i) {
+        // O += P_i V_i, V = this CTA's DV of the first d_c columns of block
+        // i's stage (MN-major)
+        if (!mbar_wait(p_full, i & 1, wc)) {
+          ok = false;
+          break;
         }
+        tc_fence_after();
+        const int st = i % NST;
+        const uint32_t va = smem_u32(sKV) + st * S::kTileBytes + vpart * (DV / 64) * S::kCBox;
+#pragma unroll
+        for (int s = 0; s < kBN / 16; ++s)
+          umma_ts(tmem + S::kTmemO, tmem + S::kTmemP + s * 8,
+                  sdesc(va + s * 2048, S::kCBox, 1024, kSw128), S::kIdescPV,
+                  (i > 0 || s > 0) ? 1u : 0u);
+        if constexpr (CL == 1)
+          umma_commit(&kv_empty[st]);
+        else
+          umma_commit_mc(&kv_empty[st], kPair);
+        umma_commit(pv_done);
       }
       if (!ok) {
         umma_commit(&mma_drain[1]);
@@ -388,14 +308,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp & 3;  // TMEM lane quarter this warp may access
     const int r = quarter * 32 + lane;
     const uint32_t t_lane = static_cast<uint32_t>(quarter * 32) << 16;
+    const int grow = row0 + r;
+    const bool row_ok = grow < p.rows;
 
-    // Q of a piece's rows: q_c as is, q_r rotated by the query position
-    // (RoPE3D), both bf16, into TMEM (q_r into shared memory when Q lives
-    // there); then q_ready.
-    auto load_q = [&](const AttnPiece& c) {
-      const int b = c.b;
-      const int grow = piece_row0(c) + r;
-      const bool row_ok = grow < p.rows;
+    // Q: q_c as is, q_r rotated by the query position (RoPE3D), both bf16.
+    {
       uint32_t w[DR / 2];
 #pragma unroll
       for (int i = 0; i < DR / 2; ++i) w[i] = 0u;
@@ -432,31 +349,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint4* qsrc = reinterpret_cast<const uint4*>(
             p.q_c + (static_cast<size_t>(b) * p.rows + (row_ok ? grow : 0)) * DC);
 #pragma unroll
-        for (int cc = 0; cc < S::kQcTmem / 64; ++cc) {
+        for (int c = 0; c < S::kQcTmem / 64; ++c) {
           uint32_t qw[32];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
-            const uint4 v = row_ok ? __ldg(qsrc + cc * 8 + i) : make_uint4(0u, 0u, 0u, 0u);
+            const uint4 v = row_ok ? __ldg(qsrc + c * 8 + i) : make_uint4(0u, 0u, 0u, 0u);
             qw[4 * i + 0] = v.x;
             qw[4 * i + 1] = v.y;
             qw[4 * i + 2] = v.z;
             qw[4 * i + 3] = v.w;
           }
-          tmem_st32(tmem + t_lane + S::kTmemQ + cc * 32, qw);
+          tmem_st32(tmem + t_lane + S::kTmemQ + c * 32, qw);
         }
       }
       if constexpr (S::kQinTmem) {
 #pragma unroll
-        for (int cc = 0; cc < DR / 32; ++cc)
-          tmem_st16(tmem + t_lane + S::kTmemQ + DC / 2 + cc * 16, w + cc * 16);
+        for (int c = 0; c < DR / 32; ++c)
+          tmem_st16(tmem + t_lane + S::kTmemQ + DC / 2 + c * 16, w + c * 16);
       } else {
         // the same 16-byte-chunk swizzle the TMA applies to the q_c part
         uint8_t* krow = sQ + S::kQKrOff + r * S::kKrRow;
 #pragma unroll
-        for (int cc = 0; cc < DR / 8; ++cc) {
-          const int phys = DR == 32 ? (cc ^ ((r >> 1) & 3)) : (cc ^ (r & 7));
+        for (int c = 0; c < DR / 8; ++c) {
+          const int phys = DR == 32 ? (c ^ ((r >> 1) & 3)) : (c ^ (r & 7));
           *reinterpret_cast<uint4*>(krow + phys * 16) =
-              make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
+              make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
         }
         fence_proxy_async_smem();
       }
@@ -465,245 +382,138 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
       }
       mbar_arrive(q_ready);
-    };
+    }
 
-    if (npc > 0) load_q(pc[0]);
     float m_run = -INFINITY;
     float l_run = 0.f;
     bool ok = true;
-    int t = 0;
-    int sk_epi = 0;  // stream-K epilogues done (phase of sk_done / sk_go)
-    for (int k = 0; ok && k < npc; ++k) {
-      const bool row_ok = piece_row0(pc[k]) + r < p.rows;
-      m_run = -INFINITY;
-      l_run = 0.f;
-      for (int j = pc[k].jb; j < pc[k].je; ++j, ++t) {
-        if (!mbar_wait(s_full, t & 1, wc)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        uint32_t sr[kBN];
-#pragma unroll
-        for (int c = 0; c < kBN / 32; ++c)
-          tmem_ld32(tmem + t_lane + S::kTmemS + c * 32,
-                    *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
-        tmem_wait_ld();
-        tc_fence_before();
-        mbar_arrive(s_free);  // S_t is in registers: the next block's scores may land
-        float sv[kBN];
-#pragma unroll
-        for (int c = 0; c < kBN; ++c) sv[c] = __uint_as_float(sr[c]);
-        const int valid = p.n_valid - j * kBN;
-        if (valid < kBN) {
-#pragma unroll
-          for (int c = 0; c < kBN; ++c)
-            if (c >= valid) sv[c] = -INFINITY;
-        }
-        // row max as 8 independent chains + a 3-level tree (short dependency path)
-        // (three-input max: two new scores per instruction)
-        float m8[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) m8[i] = sv[i];
-#pragma unroll
-        for (int c = 8; c + 16 <= kBN; c += 16)
-#pragma unroll
-          for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], sv[c + i], sv[c + 8 + i]);
-        if constexpr ((kBN - 8) % 16 != 0) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[kBN - 8 + i]);
-        }
-        const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-                               fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-        const float m_blk = mx * p.scale_log2;
-        // lazy rescale: keep the running max unless this block's max exceeds it
-        // by more than 2^8 (P <= 256 then, harmless in bf16 / fp32)
-        const bool first = j == pc[k].jb;
-        float alpha = 1.f;
-        bool need = false;
-        if (first) {
-          m_run = m_blk;
-        } else if (m_blk > m_run + kRescaleLog2) {
-          need = true;
-          alpha = ex2_approx(m_run - m_blk);
-          m_run = m_blk;
-        }
-        debug_count_rescale(need && row_ok, p.status);
-        l_run *= alpha;
-        // P_t in registers before waiting on PV_{t-1}: only the TMEM store
-        // below is serialised with the previous PV
-        const float neg_m = -m_run;
-        // scale-and-shift and the row sum two scores per instruction (paired
-        // fp32: the same IEEE roundings as the scalar forms, same 8 sum chains)
-        const uint64_t scale2 = f32x2_pack(p.scale_log2, p.scale_log2);
-        const uint64_t negm2 = f32x2_pack(neg_m, neg_m);
-        uint64_t l4[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) l4[i] = 0ull;
-        uint32_t pk[kBN / 2];
-#pragma unroll
-        for (int i = 0; i < kBN / 2; ++i) {
-          float t0, t1;
-          f32x2_unpack(f32x2_fma(f32x2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), t0, t1);
-          const float p0 = ex2_approx(t0);
-          const float p1 = ex2_approx(t1);
-          l4[i & 3] = f32x2_add(l4[i & 3], f32x2_pack(p0, p1));
-          pk[i] = pack_bf16x2(p0, p1);
-        }
-        float l8[8];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) f32x2_unpack(l4[i], l8[2 * i], l8[2 * i + 1]);
-        l_run += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
-        if (!first) {
-          // PV_{t-1} must have read P (and finished with O) before P_t is
-          // written or O is rescaled (a piece's first block: the previous
-          // piece's last PV was waited for before its epilogue)
-          if (!mbar_wait(pv_done, (t - 1) & 1, wc)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          if (__any_sync(0xffffffffu, need)) {
-#pragma unroll 1
-            for (int c = 0; c < DV / 32; ++c) {
-              uint32_t ov[32];
-              tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
-              tmem_wait_ld();
-#pragma unroll
-              for (int i = 0; i < 32; ++i)
-                ov[i] = __float_as_uint(__uint_as_float(ov[i]) * alpha);
-              tmem_st32(tmem + t_lane + S::kTmemO + c * 32, ov);
-            }
-            tmem_wait_st();
-          }
-        }
-#pragma unroll
-        for (int c = 0; c < kBN / 64; ++c)
-          tmem_st32(tmem + t_lane + S::kTmemP + c * 32,
-                    *reinterpret_cast<uint32_t(*)[32]>(&pk[c * 32]));
-        tmem_wait_st();
-        tc_fence_before();
-        mbar_arrive(p_full);
-      }
-      if (!ok) break;
-      // every score MMA of this piece has been read: the next piece's Q may
-      // replace this one's while the last PV and the epilogue run
-      if (k + 1 < npc) {
-        if constexpr (S::kQinTmem) load_q(pc[k + 1]);
-      }
-      if (!mbar_wait(pv_done, (t - 1) & 1, wc)) {
+    for (int j = 0; j < nblk; ++j) {
+      if (!mbar_wait(s_full, j & 1, wc)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      // ---------------------------------------------------------- epilogue
-      const int grow = piece_row0(pc[k]) + r;
-      if (pc[k].sk_tile < 0) {
-        const float inv_l = 1.f / l_run;
-        uint4* dst = reinterpret_cast<uint4*>(
-            p.o + (static_cast<size_t>(pc[k].b) * p.rows + grow) * DC + vpart * DV);
-#pragma unroll 1
-        for (int c = 0; c < DV / 32; ++c) {
-          uint32_t ov[32];
-          tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
-          tmem_wait_ld();
-          uint32_t pk[16];
+      uint32_t sr[kBN];
 #pragma unroll
-          for (int i = 0; i < 16; ++i)
-            pk[i] = pack_bf16x2(__uint_as_float(ov[2 * i]) * inv_l,
-                                __uint_as_float(ov[2 * i + 1]) * inv_l);
-          if (row_ok) {
+      for (int c = 0; c < kBN / 32; ++c)
+        tmem_ld32(tmem + t_lane + S::kTmemS + c * 32,
+                  *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
+      tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(s_free);  // S_j is in registers: the next block's scores may land
+      float sv[kBN];
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
-              dst[c * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-          }
-        }
-      } else {
-        // a piece of a stream-K tile: its unnormalised output and (m, l) to
-        // the workspace, row r at [chunk][r] so the warp's stores coalesce
-        const long long idx = ((static_cast<long long>(g) - p.dp_pairs) * 2 + pc[k].part) * CL + crank;
-        float4* part = p.sk_part + idx * (DV / 4) * kBM;
-#pragma unroll 1
-        for (int c = 0; c < DV / 32; ++c) {
-          uint32_t ov[32];
-          tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
-          tmem_wait_ld();
+      for (int c = 0; c < kBN; ++c) sv[c] = __uint_as_float(sr[c]);
+      const int valid = p.n_valid - j * kBN;
+      if (valid < kBN) {
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            part[(c * 8 + i) * kBM + r] =
-                make_float4(__uint_as_float(ov[4 * i]), __uint_as_float(ov[4 * i + 1]),
-                            __uint_as_float(ov[4 * i + 2]), __uint_as_float(ov[4 * i + 3]));
+        for (int c = 0; c < kBN; ++c)
+          if (c >= valid) sv[c] = -INFINITY;
+      }
+      // row max as 8 independent chains + a 3-level tree (short dependency path)
+      // (three-input max: two new scores per instruction)
+      float m8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) m8[i] = sv[i];
+#pragma unroll
+      for (int c = 8; c + 16 <= kBN; c += 16)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], sv[c + i], sv[c + 8 + i]);
+      if constexpr ((kBN - 8) % 16 != 0) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[kBN - 8 + i]);
+      }
+      const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                             fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+      const float m_blk = mx * p.scale_log2;
+      // lazy rescale: keep the running max unless this block's max exceeds it
+      // by more than 2^8 (P <= 256 then, harmless in bf16 / fp32)
+      float alpha = 1.f;
+      bool need = false;
+      if (j == 0) {
+        m_run = m_blk;
+      } else if (m_blk > m_run + kRescaleLog2) {
+        need = true;
+        alpha = ex2_approx(m_run - m_blk);
+        m_run = m_blk;
+      }
+      debug_count_rescale(need && row_ok, p.status);
+      l_run *= alpha;
+      // P_j in registers before waiting on PV_{j-1}: only the TMEM store
+      // below is serialised with the previous PV
+      const float neg_m = -m_run;
+      // scale-and-shift and the row sum two scores per instruction (paired
+      // fp32: the same IEEE roundings as the scalar forms, same 8 sum chains)
+      const uint64_t scale2 = f32x2_pack(p.scale_log2, p.scale_log2);
+      const uint64_t negm2 = f32x2_pack(neg_m, neg_m);
+      uint64_t l4[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) l4[i] = 0ull;
+      uint32_t pk[kBN / 2];
+#pragma unroll
+      for (int i = 0; i < kBN / 2; ++i) {
+        float t0, t1;
+        f32x2_unpack(f32x2_fma(f32x2_pack(sv[2 * i], sv[2 * i + 1]), scale2, negm2), t0, t1);
+        const float p0 = ex2_approx(t0);
+        const float p1 = ex2_approx(t1);
+        l4[i & 3] = f32x2_add(l4[i & 3], f32x2_pack(p0, p1));
+        pk[i] = pack_bf16x2(p0, p1);
+      }
+      float l8[8];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) f32x2_unpack(l4[i], l8[2 * i], l8[2 * i + 1]);
+      l_run += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
+      if (j > 0) {
+        // PV_{j-1} must have read P (and finished with O) before P_j is
+        // written or O is rescaled
+        if (!mbar_wait(pv_done, (j - 1) & 1, wc)) {
+          ok = false;
+          break;
         }
-        p.sk_ml[idx * 2 * kBM + r] = m_run;
-        p.sk_ml[idx * 2 * kBM + kBM + r] = l_run;
-        __threadfence();
-        const int q = pc[k].sk_tile;
-        const long long u_lo = static_cast<long long>(q) * nblk;
-        const int s_lo = sk_slot_of(u_lo, p.sk_units, p.sk_slots);
-        const int s_hi = sk_slot_of(u_lo + nblk - 1, p.sk_units, p.sk_slots);
-        // bounded mbarrier waits (not bar.sync): a thread that gave up on an
-        // earlier wait never arrives, and the others must not wait for it forever
-        mbar_arrive(sk_done);
-        if (r == 0) {
-          int last = 0;
-          if (mbar_wait(sk_done, sk_epi & 1, wc)) {
-            const int done = atomicAdd(p.sk_count + q * CL + crank, 1);
-            last = done == s_hi - s_lo;
-          }
-          *last_flag = last;
-          mbar_arrive(sk_go);
-        }
-        const bool go = mbar_wait(sk_go, sk_epi & 1, wc) && *last_flag;
-        ++sk_epi;
-        if (go) {
-          // every piece of this tile is in the workspace: combine them
-          __threadfence();
-          float wgt[8];
-          long long pidx[8];
-          const int n = min(s_hi - s_lo + 1, 8);
-          float m_max = -INFINITY;
-          for (int i = 0; i < n; ++i) {
-            const int si = s_lo + i;
-            const long long first_u = static_cast<long long>(si) * p.sk_units / p.sk_slots;
-            const int which = first_u / nblk == q ? 0 : 1;
-            pidx[i] = (static_cast<long long>(si) * 2 + which) * CL + crank;
-            wgt[i] = __ldcg(p.sk_ml + pidx[i] * 2 * kBM + r);
-            m_max = fmaxf(m_max, wgt[i]);
-          }
-          float l_tot = 0.f;
-          for (int i = 0; i < n; ++i) {
-            wgt[i] = ex2_approx(wgt[i] - m_max);
-            l_tot += wgt[i] * __ldcg(p.sk_ml + pidx[i] * 2 * kBM + kBM + r);
-          }
-          const float inv_l = 1.f / l_tot;
-          uint4* dst = reinterpret_cast<uint4*>(
-              p.o + (static_cast<size_t>(pc[k].b) * p.rows + grow) * DC + vpart * DV);
-          if (row_ok) {
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, need)) {
 #pragma unroll 1
-            for (int c = 0; c < DV / 8; ++c) {
-              float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-              for (int i = 0; i < n; ++i) {
-                const float4* src = p.sk_part + pidx[i] * (DV / 4) * kBM;
-                const float4 x0 = __ldcg(src + (2 * c) * kBM + r);
-                const float4 x1 = __ldcg(src + (2 * c + 1) * kBM + r);
-                a[0] = fmaf(wgt[i], x0.x, a[0]);
-                a[1] = fmaf(wgt[i], x0.y, a[1]);
-                a[2] = fmaf(wgt[i], x0.z, a[2]);
-                a[3] = fmaf(wgt[i], x0.w, a[3]);
-                a[4] = fmaf(wgt[i], x1.x, a[4]);
-                a[5] = fmaf(wgt[i], x1.y, a[5]);
-                a[6] = fmaf(wgt[i], x1.z, a[6]);
-                a[7] = fmaf(wgt[i], x1.w, a[7]);
-              }
-              dst[c] = make_uint4(pack_bf16x2(a[0] * inv_l, a[1] * inv_l),
-                                  pack_bf16x2(a[2] * inv_l, a[3] * inv_l),
-                                  pack_bf16x2(a[4] * inv_l, a[5] * inv_l),
-                                  pack_bf16x2(a[6] * inv_l, a[7] * inv_l));
-            }
+          for (int c = 0; c < DV / 32; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * alpha);
+            tmem_st32(tmem + t_lane + S::kTmemO + c * 32, ov);
           }
+          tmem_wait_st();
         }
       }
+#pragma unroll
+      for (int c = 0; c < kBN / 64; ++c)
+        tmem_st32(tmem + t_lane + S::kTmemP + c * 32,
+                  *reinterpret_cast<uint32_t(*)[32]>(&pk[c * 32]));
+      tmem_wait_st();
       tc_fence_before();
+      mbar_arrive(p_full);
+    }
+
+    if (ok && mbar_wait(pv_done, (nblk - 1) & 1, wc)) {
+      tc_fence_after();
+      const float inv_l = 1.f / l_run;
+      uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC +
+                                            vpart * DV);
+#pragma unroll 1
+      for (int c = 0; c < DV / 32; ++c) {
+        uint32_t ov[32];
+        tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
+        tmem_wait_ld();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          pk[i] = pack_bf16x2(__uint_as_float(ov[2 * i]) * inv_l,
+                              __uint_as_float(ov[2 * i + 1]) * inv_l);
+        if (row_ok) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            dst[c * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        }
+      }
     }
   }
 
@@ -752,57 +562,9 @@ int launch_tc(const AttnArgs& a) {
   kp.scale_log2 = a.scale_log2;
   kp.status = a.status;
   const int tiles = (a.rows + kBM - 1) / kBM;
-  // clusters per batch element: pairs of consecutive row tiles, or a split
-  // tile's two CTAs
-  const int pt_per_b = (tiles * S::kSplit + CL - 1) / CL;
-  const long long total = static_cast<long long>(pt_per_b) * a.batch;
-  kp.pt_per_b = pt_per_b;
-  kp.dp_pairs = static_cast<int>(total);
-  kp.sk_slots = 1;
-  kp.sk_units = 1;
-  kp.sk_part = nullptr;
-  kp.sk_ml = nullptr;
-  kp.sk_count = nullptr;
-  dim3 grid(pt_per_b * CL, a.batch, 1);
-  if constexpr (S::kQinTmem && S::kSplit == 1 && CL == 2) {
-    // Key-range split of the last wave: with one CTA per SM the pairs run in
-    // waves of SMs/2; when the last wave is partial, its pair tiles' key
-    // blocks are shared evenly by every pair slot of that wave (at most four
-    // slots per tile), each piece of a tile is combined by the last to finish.
-    int dev = 0, sms = 0;
-    if (a.split_ws && cudaGetDevice(&dev) == cudaSuccess &&
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
-        a.split_ws_bytes >= attention_split_workspace_bytes(DC, sms)) {
-      const int slots = sms / 2;
-      const long long full = slots > 0 ? total / slots : 0;
-      const long long rest = total - full * slots;
-      const int nblk = (a.n_valid + S::kBN - 1) / S::kBN;
-      if (full >= 1 && rest >= 1) {
-        // every slot gets at least one key block, and at most four slots share a tile
-        long long skl = rest * 4 < slots ? rest * 4 : slots;
-        if (skl > rest * nblk) skl = rest * nblk;
-        const int sk = static_cast<int>(skl);
-        unsigned char* ws = static_cast<unsigned char*>(a.split_ws);
-        const unsigned long long cnt_bytes = (static_cast<unsigned long long>(slots) * CL * 4 + 255) / 256 * 256;
-        const unsigned long long ml_bytes = static_cast<unsigned long long>(slots) * 2 * CL * 2 * kBM * 4;
-        kp.dp_pairs = static_cast<int>(full * slots);
-        kp.sk_slots = sk;
-        kp.sk_units = rest * nblk;
-        kp.sk_count = reinterpret_cast<int*>(ws);
-        kp.sk_ml = reinterpret_cast<float*>(ws + cnt_bytes);
-        kp.sk_part = reinterpret_cast<float4*>(ws + cnt_bytes + ml_bytes);
-        grid = dim3(static_cast<unsigned>((full * slots + sk) * CL), 1, 1);
-        e = cudaMemsetAsync(kp.sk_count, 0, rest * CL * sizeof(int), a.stream);
-        if (e != cudaSuccess) {
-          set_last_cuda_error(e);
-          return MLA_ERR_CUDA;
-        }
-      }
-    }
-  }
   cudaLaunchConfig_t cfg = {};
   // pairs stay within a batch row; a split tile's CTAs are adjacent
-  cfg.gridDim = grid;
+  cfg.gridDim = dim3((tiles * S::kSplit + CL - 1) / CL * CL, a.batch, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = S::kSmemBytes;
   cfg.stream = a.stream;
@@ -830,13 +592,6 @@ int launch_tc_pick(const AttnArgs& a) {
 }
 
 }  // namespace
-
-unsigned long long attention_split_workspace_bytes(int d_c, int sms) {
-  const unsigned long long slots = sms > 1 ? sms / 2 : 1;
-  const unsigned long long cnt = (slots * 2 * 4 + 255) / 256 * 256;
-  const unsigned long long per_piece = 2ull * kBM * 4 + static_cast<unsigned long long>(d_c) * kBM * 4;
-  return cnt + slots * 2 * 2 * per_piece;
-}
 
 int launch_attention_tc(const AttnArgs& a) {
   if (a.d_r == 32) {

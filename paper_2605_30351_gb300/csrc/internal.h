@@ -34,17 +34,7 @@ struct AttnArgs {
   float scale_log2;     // log2(e) / sqrt(head_dim)
   int* status;          // device status word
   cudaStream_t stream;
-  // optional caller workspace (attention_split_workspace_bytes): when given,
-  // the last, partial wave of row tiles is split over the SMs by key range
-  void* split_ws = nullptr;
-  unsigned long long split_ws_bytes = 0;
 };
-
-// Bytes of workspace the attention's key-range split needs on a device with
-// `sms` SMs for latent width d_c: a pieces-finished counter per split tile
-// and CTA, then per (slot, piece, CTA) the softmax's running max and sum
-// for 128 rows and the unnormalised [128 x d_c] fp32 output.
-unsigned long long attention_split_workspace_bytes(int d_c, int sms);
 
 // One append launch: n_tok tokens per batch element into their ring slots.
 struct AppendArgs {

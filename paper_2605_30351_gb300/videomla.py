@@ -31,7 +31,6 @@ MLA_FLAG_ROTATE_AT_USE = 4
 # Every symbol include/videomla.h declares.
 EXPORTS = ("mla_rope_table_bytes", "mla_rope_table_fill", "mla_config_check",
            "mla_cache_reset", "mla_cache_append", "mla_attention_forward",
-           "mla_attention_workspace_bytes", "mla_attention_forward_ws",
            "mla_absorb_weights", "mla_query_workspace_bytes", "mla_query_prologue",
            "mla_query_prologue_noalloc", "mla_output_projection", "mla_dense_attention_forward",
            "mla_window_workspace_bytes", "mla_attention_window_forward", "mla_decompress_window",
@@ -88,10 +87,6 @@ def load():
     lib.mla_cache_reset.argtypes = [P(mla_cache), VP]
     lib.mla_cache_append.argtypes = [P(mla_cache), VP, VP, VP, VP, VP, LL, I, VP]
     lib.mla_attention_forward.argtypes = [P(mla_cache), VP, VP, VP, I, VP, VP]
-    lib.mla_attention_workspace_bytes.argtypes = [P(mla_config), I]
-    lib.mla_attention_workspace_bytes.restype = ctypes.c_ulonglong
-    lib.mla_attention_forward_ws.argtypes = [P(mla_cache), VP, VP, VP, I, VP, ctypes.c_ulonglong,
-                                             VP, VP]
     lib.mla_status_string.argtypes = [I]
     lib.mla_status_string.restype = ctypes.c_char_p
     lib.mla_last_cuda_error.argtypes = []
@@ -113,8 +108,7 @@ def load():
     lib.mla_attention_window_forward.argtypes = [P(mla_cache), VP, VP, VP, I, VP, VP,
                                                  ctypes.c_ulonglong, VP, VP]
     for name in ("mla_rope_table_fill", "mla_config_check", "mla_cache_reset", "mla_cache_append",
-                 "mla_attention_forward", "mla_attention_forward_ws", "mla_last_cuda_error",
-                 "mla_device_status",
+                 "mla_attention_forward", "mla_last_cuda_error", "mla_device_status",
                  "mla_version", "mla_absorb_weights", "mla_query_prologue",
                  "mla_query_prologue_noalloc", "mla_output_projection",
                  "mla_dense_attention_forward", "mla_attention_window_forward",
@@ -248,31 +242,6 @@ def mla_attention_forward(cache, q_c, q_r, q_pos, o_lat, stream=None):
     _check("mla_attention_forward",
            load().mla_attention_forward(ctypes.byref(cache.struct), *args, int(Nq), out,
                                         _stream_ptr(stream)))
-
-
-def mla_attention_workspace_bytes(cfg, Nq):
-    return int(load().mla_attention_workspace_bytes(ctypes.byref(cfg), int(Nq)))
-
-
-def mla_attention_forward_ws(cache, q_c, q_r, q_pos, workspace, o_lat, stream=None):
-    """Attention with a caller workspace: the last, partial wave of row tiles
-    is split over the SMs by key range (see the C header)."""
-    cfg = cache.cfg
-    Nq = q_c.shape[1]
-    bf = torch.bfloat16
-    if not (isinstance(workspace, torch.Tensor) and workspace.is_cuda and workspace.is_contiguous()):
-        raise TypeError("workspace must be a contiguous CUDA tensor")
-    args = (
-        _dev(q_c, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "q_c"),
-        _dev(q_r, bf, (cfg.batch, Nq, cfg.heads, cfg.d_r), "q_r"),
-        _dev(q_pos, torch.int32, (cfg.batch, Nq, 3), "q_pos"),
-    )
-    out = _dev(o_lat, bf, (cfg.batch, Nq, cfg.heads, cfg.d_c), "o_lat")
-    _check("mla_attention_forward_ws",
-           load().mla_attention_forward_ws(ctypes.byref(cache.struct), *args, int(Nq),
-                                           ctypes.c_void_p(workspace.data_ptr()),
-                                           workspace.numel() * workspace.element_size(), out,
-                                           _stream_ptr(stream)))
 
 
 def mla_window_workspace_bytes(cfg, Nq):
