@@ -91,8 +91,8 @@ def kernel_source_hash(name):
 
 def append_kernel_name(w):
     """The append kernel the library launches for this shape: a cluster of
-    d_c/64 CTAs per token tile when those CTAs fit in one wave, else one CTA
-    per tile (the launch also checks that the clusters are co-resident)."""
+    d_c/64 CTAs per token tile when those CTAs fit in one wave (the launch
+    also checks that the clusters are co-resident), else one CTA per tile."""
     tiles = -(-w.chunk_tokens // 128)
     sms = torch.cuda.get_device_properties(0).multi_processor_count if torch.cuda.is_available() else 152
     if 128 <= w.d_c <= 256 and tiles * w.batch * (w.d_c // 64) <= sms:

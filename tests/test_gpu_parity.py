@@ -632,3 +632,4 @@ def test_host_and_pinned_memory_refused():
     assert rc == V.MLA_ERR_ARG
     V.mla_attention_forward(cache, *dev, o)           # the same call on device memory runs
     torch.cuda.synchronize()
+
