@@ -141,6 +141,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   // every CTA's barriers must be initialised before a peer's multicast lands
   if constexpr (CL > 1) cluster_sync();
+  grid_dep_sync();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -501,13 +502,15 @@ int launch_tc(const AppendArgs& a) {
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = a.stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = cluster ? kCl : 1;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_sync
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   e = cudaLaunchKernelEx(&cfg, kern, tm_x, tm_wc, tm_wk, kp);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {

@@ -178,6 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   // the peer's barriers must be initialised before any multicast lands
   if constexpr (CL > 1) cluster_sync();
+  grid_dep_sync();
   const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
 
   if (warp == 0) {
@@ -568,13 +569,15 @@ int launch_tc(const AttnArgs& a) {
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = S::kSmemBytes;
   cfg.stream = a.stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = CL;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_sync
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   e = cudaLaunchKernelEx(&cfg, kern, tm_qc, tm_c, tm_kr, kp);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {

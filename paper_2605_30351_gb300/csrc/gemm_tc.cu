@@ -99,6 +99,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  grid_dep_sync();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -234,9 +235,18 @@ int launch_gemm(const void* a, const void* b, int M, int N, int K, GemmKParams k
   kp.M = M;
   kp.N = N;
   kp.K = K;
-  const dim3 grid((M + kBM - 1) / kBM, (N + BN - 1) / BN);
-  kern<<<grid, kThreads, S::kSmemBytes, stream>>>(tm_a, tm_b, kp);
-  e = cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((M + kBM - 1) / kBM, (N + BN - 1) / BN);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = S::kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_sync
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, tm_a, tm_b, kp);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return MLA_ERR_CUDA;

@@ -61,6 +61,19 @@ __device__ __forceinline__ void debug_count_rescale(bool rescaled, int* status) 
 #endif
 }
 
+// Programmatic dependent launch. The library's kernels are launched with
+// programmatic stream serialization, so their CTAs may start while the
+// previous kernel in the stream is still running. Before grid_dep_sync() a
+// kernel only does set-up that touches no global memory (barrier init, TMEM
+// allocation, cluster sync); grid_dep_sync() lets the next kernel in the
+// stream launch once every CTA of this one has started, then waits until the
+// previous kernel has completed and its writes are visible. Every thread
+// calls it before its first global-memory access.
+__device__ __forceinline__ void grid_dep_sync() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 // ----------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)

@@ -53,6 +53,7 @@ __global__ void __launch_bounds__(kThreads)
                            uint4* __restrict__ kr_rot, int* __restrict__ q_local, int batch,
                            int nq, int slots, int n_valid, int T, int W, int S, int pairs,
                            long long fw, int rope_len, int pairs_t, int pairs_h, int* status) {
+  grid_dep_sync();
   // local time of the frame held in each frame slot (-1: none), once per block
   __shared__ int t_of_slot[kMaxFrames];
   for (int j = threadIdx.x; j < W && j < kMaxFrames; j += kThreads)
@@ -121,12 +122,21 @@ int launch_window_assemble(const WindowArgs& a) {
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const long long want = (n_all + kThreads - 1) / kThreads;
   const int blocks = static_cast<int>(want < 8ll * sms ? want : 8ll * sms);
-  window_assemble_kernel<<<blocks, kThreads, 0, a.stream>>>(
-      static_cast<const uint4*>(a.kr), a.q_pos, reinterpret_cast<const int2*>(a.frame_hw),
-      reinterpret_cast<const float2*>(a.rope), static_cast<uint4*>(a.kr_rot), a.q_pos_local,
-      a.batch, a.nq, a.slots, a.n_valid, a.T, a.W, a.S, pairs, a.frames_written, a.rope_len,
-      a.pairs_t, a.pairs_h, a.status);
-  const cudaError_t e = cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(blocks, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = a.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_sync
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(
+      &cfg, window_assemble_kernel, static_cast<const uint4*>(a.kr), a.q_pos,
+      reinterpret_cast<const int2*>(a.frame_hw), reinterpret_cast<const float2*>(a.rope),
+      static_cast<uint4*>(a.kr_rot), a.q_pos_local, a.batch, a.nq, a.slots, a.n_valid, a.T, a.W,
+      a.S, pairs, a.frames_written, a.rope_len, a.pairs_t, a.pairs_h, a.status);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return MLA_ERR_CUDA;
