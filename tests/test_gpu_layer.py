@@ -76,6 +76,41 @@ def test_query_prologue_matches_oracle(nq, batch, shape):
     assert_close(f64(q_r), ref_qr, what="q_r")
 
 
+def test_layer_gemms_at_four_chunks_match_oracle():
+    """Four Wan-1.3B chunks (18,720 query tokens): both query-prologue GEMMs and
+    the output projection take 256-wide tiles as paired-SM MMAs (two M tiles
+    per M = 256 MMA, each CTA holding half of the B rows; 147 M tiles, so the
+    last pair has a tile past the tokens). Sampled rows, including the first
+    and last pair, against the oracle (Eqs. cq, qnope, qrope, absorb-v)."""
+    w = synth.workload("wan", batch=4)
+    nq = w.chunk_tokens
+    wt = synth.draw_layer_weights(w, seed=74)
+    dev = {k: v.cuda() for k, v in wt.items()}
+    cfg = V.make_config(w)
+    w_qcat, w_b = V.mla_absorb_weights(cfg, dev["w_uq"], dev["w_uk"], dev["w_qr"], dev["gamma_q"],
+                                       dev["w_uv"], dev["w_o"])
+    x = synth.draw_tokens(w, nq, 75)
+    ws = torch.empty(V.mla_query_workspace_bytes(cfg, nq), dtype=torch.uint8, device="cuda")
+    q_c = torch.empty(4, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    q_r = torch.empty(4, nq, w.heads, w.d_r, dtype=torch.bfloat16, device="cuda")
+    V.mla_query_prologue(cfg, x.cuda(), dev["w_dq"], w_qcat, ws, q_c, q_r)
+    o = synth.draw_queries(w, nq, 76)[0]          # any bf16 latent output [4, nq, H, d_c]
+    y = torch.empty(4, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
+    V.mla_output_projection(cfg, o.cuda(), w_b, y)
+    torch.cuda.synchronize()
+    w64 = weights64(wt)
+    B = O.absorbed_output_matrices(w64["w_uv"], w64["w_o"])            # [H, d, d_c]
+    for b, toks in ((0, [0, 1, 127, 128, 255, 256, 2000]), (3, [4000, 4607, 4608, 4679])):
+        xs = f64(x[b])[toks]
+        c_q = O.rmsnorm(xs @ w64["w_dq"].T, w64["gamma_q"], w.rms_eps)
+        assert_close(f64(q_c[b])[toks], O.absorb_query(c_q, w64["w_uq"], w64["w_uk"]),
+                     what=f"q_c, chunk {b}")
+        assert_close(f64(q_r[b])[toks], np.einsum("hrq,nq->nhr", w64["w_qr"], c_q),
+                     what=f"q_r, chunk {b}")
+        ref_y = np.einsum("hdc,nhc->nd", B, f64(o[b])[toks])
+        assert_close(f64(y[b])[toks], ref_y, what=f"y, chunk {b}")
+
+
 def test_full_layer_output_matches_non_absorbed_oracle():
     """x -> cache append (every window frame) -> query prologue -> latent
     attention -> output projection on the GPU, against the oracle's
