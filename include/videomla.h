@@ -263,7 +263,8 @@ unsigned long long mla_query_workspace_bytes(const mla_config* cfg, int Nq);
  *             bytes, 16-byte aligned, owned by the caller; its contents are
  *             scratch between the two GEMMs of this call
  *  q_c     bf16 [batch][Nq][H][d_c];  q_r bf16 [batch][Nq][H][d_r] (unrotated)
- * MLA_ERR_UNSUPPORTED unless d_q and hidden are multiples of 64.
+ * MLA_ERR_UNSUPPORTED unless d_q and hidden are multiples of 64 and
+ * batch * Nq <= 8,388,352 (65,534 tiles of 128 query tokens).
  */
 int mla_query_prologue(const mla_config* cfg, const void* x, const void* w_dq,
                        const void* w_qcat, int Nq, void* workspace,
@@ -299,7 +300,8 @@ int mla_query_prologue_noalloc(const mla_config* cfg, const void* x, const void*
  * Output projection of the latent attention output (Eq. absorb-v):
  *     y = sum_h B_h o_lat,h = o_lat W_B^T
  *  o_lat bf16 [batch][Nq][H][d_c], w_b bf16 [hidden][H*d_c],
- *  y bf16 [batch][Nq][hidden]. MLA_ERR_UNSUPPORTED unless H*d_c % 64 == 0.
+ *  y bf16 [batch][Nq][hidden]. MLA_ERR_UNSUPPORTED unless H*d_c % 64 == 0 and
+ *  batch * Nq <= 8,388,352 (65,534 tiles of 128 tokens).
  */
 int mla_output_projection(const mla_config* cfg, const void* o_lat, const void* w_b, int Nq,
                           void* y, void* stream);

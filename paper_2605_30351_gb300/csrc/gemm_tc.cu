@@ -86,8 +86,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * kBM;
-  const int n0 = blockIdx.y * BN;
+  // N tiles run fastest (blockIdx.x), so the N tiles of one row tile of A
+  // follow one another and A comes from HBM once; B stays in L2. PAIR: the
+  // two CTAs of an x-cluster take M tiles 2y and 2y + 1 of the same N tile.
+  const int n_tile = PAIR ? blockIdx.x / 2 : blockIdx.x;
+  const int m0 = (PAIR ? 2 * blockIdx.y + (blockIdx.x & 1) : blockIdx.y) * kBM;
+  const int n0 = n_tile * BN;
   const int k_blocks = p.K / kBK;
   const WaitCtx wc{abort_flag, p.status};
 
@@ -134,15 +138,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (crank == 0) mbar_arrive_expect_tx(&full[st], S::kTxBytes);
           tma_load_2d_pair(a, &tm_a, bar, kb * kBK, m0);
           tma_load_2d_pair(a + S::kABytes, &tm_b, bar, kb * kBK, n0 + crank * S::kBBox);
-          issued = kb + 1;
-          continue;
-        }
-        mbar_arrive_expect_tx(&full[st], S::kStageBytes);
-        tma_load_2d(a, &tm_a, &full[st], kb * kBK, m0);
+        } else {
+          mbar_arrive_expect_tx(&full[st], S::kTxBytes);
+          tma_load_2d(a, &tm_a, &full[st], kb * kBK, m0);
 #pragma unroll
-        for (int h = 0; h < S::kHalves; ++h)
-          tma_load_2d(a + S::kABytes + h * S::kBN1 * 128, &tm_b, &full[st], kb * kBK,
-                      n0 + h * S::kBN1);
+          for (int h = 0; h < S::kHalves; ++h)
+            tma_load_2d(a + S::kABytes + h * S::kBN1 * 128, &tm_b, &full[st], kb * kBK,
+                        n0 + h * S::kBN1);
+        }
         issued = kb + 1;
       }
       if constexpr (PAIR) {
@@ -174,16 +177,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_pair_ss(tmem, sdesc(aa + k * 32, 16, 1024, kSw128),
                          sdesc(ba + k * 32, 16, 1024, kSw128), S::kIdesc, (kb | k) != 0 ? 1u : 0u);
           umma_pair_commit_mc(&empty[st], 3);
-          continue;
+        } else {
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+#pragma unroll
+            for (int h = 0; h < S::kHalves; ++h)
+              umma_ss(tmem + h * S::kBN1, sdesc(aa + k * 32, 16, 1024, kSw128),
+                      sdesc(ba + h * S::kBN1 * 128 + k * 32, 16, 1024, kSw128), S::kIdesc,
+                      (kb | k) != 0 ? 1u : 0u);
+          umma_commit(&empty[st]);
         }
-#pragma unroll
-        for (int k = 0; k < kBK / 16; ++k)
-#pragma unroll
-          for (int h = 0; h < S::kHalves; ++h)
-            umma_ss(tmem + h * S::kBN1, sdesc(aa + k * 32, 16, 1024, kSw128),
-                    sdesc(ba + h * S::kBN1 * 128 + k * 32, 16, 1024, kSw128), S::kIdesc,
-                    (kb | k) != 0 ? 1u : 0u);
-        umma_commit(&empty[st]);
       }
       if constexpr (PAIR)
         umma_pair_commit_mc(acc_full, 3);
@@ -233,7 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
       if constexpr (EPI == kStoreSq)
-        if (m < p.M) p.sq[static_cast<size_t>(blockIdx.y) * p.M + m] = ss_own;
+        if (m < p.M) p.sq[static_cast<size_t>(n_tile) * p.M + m] = ss_own;
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
     if (have_acc) {
@@ -289,14 +292,16 @@ int launch_gemm(const void* a, const void* b, int M, int N, int K, GemmKParams k
   // PAIR: M tiles rounded up to pairs (a last tile past M loads zeros and
   // stores nothing)
   const int m_tiles = (M + kBM - 1) / kBM;
-  cfg.gridDim = dim3(PAIR ? (m_tiles + 1) / 2 * 2 : m_tiles, (N + BN - 1) / BN);
+  if (m_tiles > 65534) return MLA_ERR_UNSUPPORTED;  // row tiles index the grid's y dimension
+  const int n_tiles = (N + BN - 1) / BN;
+  cfg.gridDim = PAIR ? dim3(2 * n_tiles, (m_tiles + 1) / 2) : dim3(n_tiles, m_tiles);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = S::kSmemBytes;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_sync
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].id = cudaLaunchAttributeClusterDimension;  // PAIR: M tiles 2y, 2y + 1
   attr[1].val.clusterDim.x = PAIR ? 2 : 1;
   attr[1].val.clusterDim.y = 1;
   attr[1].val.clusterDim.z = 1;
