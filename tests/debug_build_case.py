@@ -3,7 +3,8 @@ named on the command line (release or debug build), runs a fixed set of
 calls (append + attention on the 21-frame ring, the sink window, the
 decompression, the query prologue and output projection; the append's
 cluster and split forms and the split-output attention at d_c = 256 and 512;
-the online softmax's rescale branch in the absorbed and dense kernels) on
+the layer GEMMs' paired-SM form at four chunks; the online softmax's
+rescale branch in the absorbed and dense kernels) on
 seeded inputs and saves every output, the device status word and the debug
 build's count of softmax rescales (-1 for the release build, which does not
 count)."""
@@ -83,6 +84,23 @@ def main(lib_path, out_path):
                                 o)
         torch.cuda.synchronize()
         out[f"c_{d_c}"], out[f"kr_{d_c}"], out[f"o_{d_c}"] = cache.c.cpu(), cache.kr.cpu(), o.cpu()
+    # the layer GEMMs in their paired-SM form (four Wan chunks: 147 row tiles,
+    # the last pair half past the tokens)
+    w = synth.workload("wan", batch=4)
+    cfg = V.make_config(w)
+    wt = {k: t.cuda() for k, t in synth.draw_layer_weights(w, 37).items()}
+    w_qcat, w_b = V.mla_absorb_weights(cfg, wt["w_uq"], wt["w_uk"], wt["w_qr"], wt["gamma_q"],
+                                       wt["w_uv"], wt["w_o"])
+    nq = w.chunk_tokens
+    x = synth.draw_tokens(w, nq, 87).cuda()
+    wsq = torch.empty(V.mla_query_workspace_bytes(cfg, nq), dtype=torch.uint8, device="cuda")
+    qc4 = torch.empty(4, nq, w.heads, w.d_c, dtype=torch.bfloat16, device="cuda")
+    qr4 = torch.empty(4, nq, w.heads, w.d_r, dtype=torch.bfloat16, device="cuda")
+    V.mla_query_prologue(cfg, x, wt["w_dq"], w_qcat, wsq, qc4, qr4)
+    y4 = torch.empty(4, nq, w.hidden, dtype=torch.bfloat16, device="cuda")
+    V.mla_output_projection(cfg, qc4, w_b, y4)
+    torch.cuda.synchronize()
+    out["q_c4"], out["q_r4"], out["y4"] = qc4.cpu(), qr4.cpu(), y4.cpu()
     # the online softmax's rescale branch: a dominant key in the last key
     # block for a third of the rows, absorbed (390 keys) and dense (500 keys)
     from test_gpu_softmax import absorbed_inputs, dense_inputs
