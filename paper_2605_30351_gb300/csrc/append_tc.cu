@@ -63,9 +63,11 @@ struct AppendShape {
   // [CL][128] partial sums of squares at the front of shared memory: the same
   // offset in every CTA of a cluster, whichever slice it computes
   static constexpr int kRedOff = CL > 1 ? (CL * kBM * 4 + 1023) / 1024 * 1024 : 0;
-  static constexpr int kFit = (232448 - 1024 - kBarBytes - kRedOff) / kStageBytes;
+  // this CTA's gamma columns, fetched by the epilogue warps during the K loop
+  static constexpr int kGammaBytes = NC * 2;
+  static constexpr int kFit = (232448 - 1024 - kBarBytes - kGammaBytes - kRedOff) / kStageBytes;
   static constexpr int kStages = kFit > 6 ? 6 : kFit;
-  static constexpr int kSmemBytes = 1024 + kRedOff + kStages * kStageBytes + kBarBytes;
+  static constexpr int kSmemBytes = 1024 + kRedOff + kStages * kStageBytes + kBarBytes + kGammaBytes;
   static constexpr uint32_t kTmemCols = N <= 32 ? 32 : (N <= 64 ? 64 : (N <= 256 ? 256 : 512));
   // output staging row: N bf16 plus 16 bytes, so rows start on different banks
   static constexpr int kOutStride = N * 2 + 16;
@@ -237,6 +239,41 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     const uint32_t t_row = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int n = row0 + r;
     const bool row_ok = n < p.n_tok;
+    // What the epilogue reads from global memory is fetched while the MMAs
+    // run, so that no load latency follows the accumulator: this CTA's gamma
+    // columns into shared memory (read by every row), the row's ring slot
+    // and its RoPE factors (cos, sin per pair) into registers.
+    uint4* gamma_s = reinterpret_cast<uint4*>(smem + NST * S::kStageBytes + S::kBarBytes);
+    for (int i = threadIdx.x - 64; i < NC / 8; i += 128)
+      gamma_s[i] = p.gamma ? __ldg(reinterpret_cast<const uint4*>(p.gamma + c0) + i)
+                           : make_uint4(0x3f803f80u, 0x3f803f80u, 0x3f803f80u, 0x3f803f80u);
+    const long long f = p.first_frame + n / p.T;
+    const long long slot_n = frame_base_slot(f, p.T, p.W, p.S) + n % p.T;
+    const long long my_slot =
+        row_ok && debug_in_range(slot_n, 0, p.slots, p.status) ? slot_n : -1;
+    float2 cs[NK > 0 ? NK / 2 : 1];
+    if constexpr (NK > 0) {
+      int pa[3] = {0, 0, 0};
+      if (row_ok && p.rotate) {
+        const int* pp = p.pos + (static_cast<size_t>(b) * p.n_tok + n) * 3;
+        pa[0] = __ldg(pp);
+        pa[1] = __ldg(pp + 1);
+        pa[2] = __ldg(pp + 2);
+#pragma unroll
+        for (int a = 0; a < 3; ++a)
+          if (pa[a] < 0 || pa[a] >= p.rope_len) {
+            record_status(p.status, MLA_ERR_RANGE);
+            pa[a] = 0;
+          }
+      }
+#pragma unroll
+      for (int pr = 0; pr < NK / 2; ++pr) {
+        const int ps = pr < p.pairs_t ? pa[0] : (pr < p.pairs_t + p.pairs_h ? pa[1] : pa[2]);
+        cs[pr] = p.rotate ? __ldg(p.rope + static_cast<size_t>(ps) * (DR / 2) + pr)
+                          : make_float2(1.f, 0.f);
+      }
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // gamma_s is complete
     const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
     // The finished bf16 rows are staged in shared memory (the stage ring is
     // free once the accumulator is complete) and then written out by all 128
@@ -274,9 +311,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     }
     if (have_acc) {
       const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
-      const long long f = p.first_frame + n / p.T;
-      const long long slot = frame_base_slot(f, p.T, p.W, p.S) + n % p.T;
-      slot_of[r] = row_ok && debug_in_range(slot, 0, p.slots, p.status) ? slot : -1;
+      slot_of[r] = my_slot;
       uint8_t* srow = stage_out + r * S::kOutStride;
       // pass 2: gamma * c / rms -> bf16
 #pragma unroll 1
@@ -287,8 +322,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
         uint32_t gw[16];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          uint4 g4 = make_uint4(0x3f803f80u, 0x3f803f80u, 0x3f803f80u, 0x3f803f80u);  // ones
-          if (p.gamma) g4 = __ldg(reinterpret_cast<const uint4*>(p.gamma + c0 + cb * 32) + i);
+          const uint4 g4 = gamma_s[cb * 4 + i];
           gw[4 * i] = g4.x; gw[4 * i + 1] = g4.y; gw[4 * i + 2] = g4.z; gw[4 * i + 3] = g4.w;
         }
         uint32_t pk[16];
@@ -302,20 +336,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
       // positional key: RoPE3D at the token's (t, h, w), or unrotated
-      int pa[3] = {0, 0, 0};
-      if (NK > 0 && row_ok && p.rotate) {
-        const int* pp = p.pos + (static_cast<size_t>(b) * p.n_tok + n) * 3;
-        pa[0] = __ldg(pp);
-        pa[1] = __ldg(pp + 1);
-        pa[2] = __ldg(pp + 2);
 #pragma unroll
-        for (int a = 0; a < 3; ++a)
-          if (pa[a] < 0 || pa[a] >= p.rope_len) {
-            record_status(p.status, MLA_ERR_RANGE);
-            pa[a] = 0;
-          }
-      }
-#pragma unroll 1
       for (int cb = 0; cb < NK / 32; ++cb) {
         uint32_t v[32];
         tmem_ld32(t_row + NC + cb * 32, v);
@@ -323,11 +344,9 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
         uint32_t pk[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const int pr = cb * 16 + i;
-          const int ps = pr < p.pairs_t ? pa[0] : (pr < p.pairs_t + p.pairs_h ? pa[1] : pa[2]);
-          const float2 cs = __ldg(p.rope + static_cast<size_t>(ps) * (DR / 2) + pr);
+          const float2 f2 = cs[cb * 16 + i];
           const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
-          pk[i] = p.rotate ? pack_bf16x2(x0 * cs.x - x1 * cs.y, x0 * cs.y + x1 * cs.x)
+          pk[i] = p.rotate ? pack_bf16x2(x0 * f2.x - x1 * f2.y, x0 * f2.y + x1 * f2.x)
                            : pack_bf16x2(x0, x1);
         }
 #pragma unroll
