@@ -9,16 +9,19 @@
 //              K step at the paper's shape).
 //   warps 2-5  epilogue, thread i = token i: RMSNorm over the d_c columns in
 //              fp32, gamma, RoPE3D on the d_r columns (skipped when the
-//              cache keeps k^R unrotated), bf16, 16-byte stores into the
-//              token's slot: (f mod W) * T + k, or with S sink frames f * T + k
-//              for f < S and (S + (f - S) mod (W - S)) * T + k after them.
+//              cache keeps k^R unrotated), bf16, staged in shared memory and
+//              bulk-copied into the token's slot: (f mod W) * T + k, or with S
+//              sink frames f * T + k for f < S and (S + (f - S) mod (W - S)) * T
+//              + k after them.
 // For d_c = 512 the [128 x (d_c + d_r)] accumulator does not fit the 512
 // TMEM columns; the launch then runs two CTAs per token tile (blockIdx.z):
 // one accumulates c (two N = 256 MMAs per K step) and applies RMSNorm, the
 // other accumulates k^R and applies RoPE. Both stream the same x tile.
 // When one CTA per token tile would leave most SMs idle (one chunk at batch
 // 1), a cluster of d_c/64 CTAs shares each token tile, one per 64 columns of
-// c (see AppendShape).
+// c (see AppendShape). When the tiles exceed one wave, two CTAs with fewer
+// stages share each SM, so that one's start-up and epilogue overlap the
+// other's K loop.
 #include <cmath>
 #include <type_traits>
 
@@ -31,6 +34,10 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kThreads = 192;
+// dynamic shared memory of a CTA that has an SM to itself, and of one of two
+// CTAs sharing an SM (228 KB per SM, 1 KB of it reserved per CTA)
+constexpr int kSmemOne = 232448;
+constexpr int kSmemHalf = (233472 - 2 * 1024) / 2;
 
 // What one CTA computes: NC columns of c, from column c0 (given at run time),
 // and NK columns of k^R, into one [128 x (NC + NK)] TMEM accumulator:
@@ -44,7 +51,7 @@ constexpr int kThreads = 192;
 //    share of the weights. The CTAs share each x box through TMA multicast
 //    (each fetches a part of it from L2 for all) and exchange their partial
 //    RMSNorm sums of squares through distributed shared memory.
-template <int DC, int DR, int NC, int NK, int CL = 1>
+template <int DC, int DR, int NC, int NK, int CL = 1, int BUDGET = kSmemOne>
 struct AppendShape {
   static constexpr int N = NC + NK;
   static constexpr bool kSplitN = N > 256;  // then MMAs of at most 256: c part(s), k part
@@ -65,13 +72,14 @@ struct AppendShape {
   static constexpr int kRedOff = CL > 1 ? (CL * kBM * 4 + 1023) / 1024 * 1024 : 0;
   // this CTA's gamma columns, fetched by the epilogue warps during the K loop
   static constexpr int kGammaBytes = NC * 2;
-  static constexpr int kFit = (232448 - 1024 - kBarBytes - kGammaBytes - kRedOff) / kStageBytes;
+  static constexpr int kFit = (BUDGET - 1024 - kBarBytes - kGammaBytes - kRedOff) / kStageBytes;
   static constexpr int kStages = kFit > 6 ? 6 : kFit;
   static constexpr int kSmemBytes = 1024 + kRedOff + kStages * kStageBytes + kBarBytes + kGammaBytes;
   static constexpr uint32_t kTmemCols = N <= 32 ? 32 : (N <= 64 ? 64 : (N <= 256 ? 256 : 512));
   // output staging row: N bf16 plus 16 bytes, so rows start on different banks
   static constexpr int kOutStride = N * 2 + 16;
   static_assert(kBM * kOutStride + kBM * 8 <= kStages * kStageBytes, "staging fits in the ring");
+  static_assert(kOutStride % 16 == 0 && (NC * 2) % 16 == 0, "bulk copies need 16-byte rows");
   static_assert(DC % 32 == 0 && DR % 32 == 0 && DR <= 64 && (DC <= 256 || DC % 256 == 0),
                 "shape");
   static_assert(N > 0 && NC % 32 == 0 && (NK == 0 || NK == DR), "parts");
@@ -98,11 +106,11 @@ struct AppendKParams {
 };
 
 // tile: the token tile (128 tokens) of this CTA; c0: its first column of c
-template <int DC, int DR, int NC, int NK, int CL>
+template <int DC, int DR, int NC, int NK, int CL, int BUDGET = kSmemOne>
 __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUtensorMap* tm_wc,
                                             const CUtensorMap* tm_wk, const AppendKParams& p,
                                             int tile, int c0) {
-  using S = AppendShape<DC, DR, NC, NK, CL>;
+  using S = AppendShape<DC, DR, NC, NK, CL, BUDGET>;
   constexpr int NST = S::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = align_smem_1024(smem_raw);
@@ -275,12 +283,16 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");  // gamma_s is complete
     const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
-    // The finished bf16 rows are staged in shared memory (the stage ring is
-    // free once the accumulator is complete) and then written out by all 128
-    // threads together, so that consecutive threads store consecutive 16-byte
-    // pieces of a row instead of each thread writing its own row.
-    uint8_t* stage_out = smem;                                   // [128][kOutStride]
-    long long* slot_of = reinterpret_cast<long long*>(smem + kBM * S::kOutStride);  // [128]
+    // Each thread stages its finished bf16 row in shared memory (the stage
+    // ring is free once the accumulator is complete). One CTA per tile then
+    // hands each row to the bulk-copy engine, one copy for its c columns and
+    // one for k^R: at the Wan shape ~1.9 us per tile, against ~2.9 us for
+    // per-thread 16-byte stores of whole rows and ~3.4 us for a coalesced
+    // store loop of the four warps after a barrier. A cluster's CTAs hold
+    // 64-column slices, whose 128-byte rows the coalesced loop writes faster
+    // than 256 small copies.
+    uint8_t* stage_out = smem;                                                     // [128][kOutStride]
+    long long* slot_of = reinterpret_cast<long long*>(smem + kBM * S::kOutStride);  // [128], clusters
     // pass 1: sum of squares of this CTA's c columns (fp32)
     float ss = 0.f;
     if (have_acc) {
@@ -311,7 +323,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     }
     if (have_acc) {
       const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
-      slot_of[r] = my_slot;
+      if constexpr (CL > 1) slot_of[r] = my_slot;
       uint8_t* srow = stage_out + r * S::kOutStride;
       // pass 2: gamma * c / rms -> bf16
 #pragma unroll 1
@@ -355,22 +367,39 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
               make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
       }
     }
-    // the four epilogue warps only
-    asm volatile("bar.sync 1, 128;" ::: "memory");
-    if (have_acc) {
-      constexpr int kChunks = S::N * 2 / 16;  // 16-byte pieces per output row
-      constexpr int kChunksC = NC * 2 / 16;
-      for (int q = r; q < kBM * kChunks; q += kBM) {
-        const int row = q / kChunks, ch = q % kChunks;
-        const long long slot = slot_of[row];
-        if (slot < 0) continue;
-        const uint4 v = *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
-        if (ch < kChunksC)
-          *reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC + c0 +
-                                    ch * 8) = v;
-        else
-          *reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR +
-                                    (ch - kChunksC) * 8) = v;
+    if constexpr (CL == 1) {
+      if (have_acc && my_slot >= 0) {
+        // the row's slot: c at (b * slots + slot) * d_c + c0, k^R at
+        // (b * slots + slot) * d_r; both 16-byte aligned (d_c, d_r, c0 are
+        // multiples of 32), as is the staged row (kOutStride is)
+        const uint8_t* srow = stage_out + r * S::kOutStride;
+        const size_t row_id = static_cast<size_t>(b) * p.slots + my_slot;
+        fence_proxy_async_smem();
+        if constexpr (NC > 0) bulk_store(p.c + row_id * DC + c0, srow, NC * 2);
+        if constexpr (NK > 0) bulk_store(p.kr + row_id * DR, srow + NC * 2, NK * 2);
+        bulk_commit();
+        bulk_wait_read_all();  // the staging rows must outlive the copies' reads
+      }
+    } else {
+      // the four epilogue warps only: consecutive threads store consecutive
+      // 16-byte pieces of the staged rows
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (have_acc) {
+        constexpr int kChunks = S::N * 2 / 16;  // 16-byte pieces per output row
+        constexpr int kChunksC = NC * 2 / 16;
+        for (int q = r; q < kBM * kChunks; q += kBM) {
+          const int row = q / kChunks, ch = q % kChunks;
+          const long long slot = slot_of[row];
+          if (slot < 0) continue;
+          const uint4 v =
+              *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
+          if (ch < kChunksC)
+            *reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC +
+                                      c0 + ch * 8) = v;
+          else
+            *reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR +
+                                      (ch - kChunksC) * 8) = v;
+        }
       }
     }
   }
@@ -389,6 +418,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                          const __grid_constant__ CUtensorMap tm_wc,
                          const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
   append_body<DC, DR, DC, DR, 1>(&tm_x, &tm_wc, &tm_wk, p, blockIdx.x, 0);
+}
+
+// Grids of more than one wave: two CTAs share each SM (fewer stages each), so
+// that one CTA's start-up and epilogue run under the other's K loop.
+template <int DC, int DR>
+__global__ void __launch_bounds__(kThreads, 2)
+    mla_append_tc_kernel_x2(const __grid_constant__ CUtensorMap tm_x,
+                            const __grid_constant__ CUtensorMap tm_wc,
+                            const __grid_constant__ CUtensorMap tm_wk, const AppendKParams p) {
+  append_body<DC, DR, DC, DR, 1, kSmemHalf>(&tm_x, &tm_wc, &tm_wk, p, blockIdx.x, 0);
 }
 
 // d_c > 256: blockIdx.z = 0 computes c, 1 computes k^R, for the same tokens
@@ -466,6 +505,12 @@ int launch_tc(const AppendArgs& a) {
       cluster = clusters <= resident;
     }
   }
+  // two CTAs per SM when the grid has more than one wave of single CTAs and
+  // two stages of the unsplit form fit in half an SM's shared memory
+  constexpr int kStageX2 = kBM * kBK * 2 + (DC + DR) * kBK * 2;
+  constexpr bool kX2Fits = !kSplit && DC + DR <= 256 &&  // two 256-column TMEM accumulators
+                           (kSmemHalf - 1024 - 256 - DC * 2) / kStageX2 >= 2;
+  const bool x2 = kX2Fits && !cluster && static_cast<long long>(tiles) * a.batch > sms;
   // shapes of the CTAs each form launches (d_c > 256: the c and k^R halves;
   // the cluster form: a 64-column c slice and k^R; else both parts)
   using S = AppendShape<DC, DR, DC, kSplit ? 0 : DR>;
@@ -474,7 +519,9 @@ int launch_tc(const AppendArgs& a) {
   using SCk = std::conditional_t<kClusterable, AppendShape<DC, DR, 64, DR, kCl>, S>;
   constexpr int kSmemPlain = S::kSmemBytes > SK::kSmemBytes ? S::kSmemBytes : SK::kSmemBytes;
   constexpr int kSmemCl = SCc::kSmemBytes > SCk::kSmemBytes ? SCc::kSmemBytes : SCk::kSmemBytes;
-  const int smem = cluster ? kSmemCl : kSmemPlain;
+  int smem = cluster ? kSmemCl : kSmemPlain;
+  if constexpr (kX2Fits)
+    if (x2) smem = AppendShape<DC, DR, DC, DR, 1, kSmemHalf>::kSmemBytes;
   CUtensorMap tm_x, tm_wc, tm_wk;
   const unsigned long long H = a.hidden, n_tok = a.n_tok;
   if (!encode_map_3d_bf16(&tm_x, a.x, H, n_tok, a.batch, H * 2, n_tok * H * 2, kBK,
@@ -491,6 +538,8 @@ int launch_tc(const AppendArgs& a) {
     kern = cluster ? mla_append_tc_cluster_kernel<DC, DR> : mla_append_tc_kernel<DC, DR>;
   else
     kern = mla_append_tc_kernel<DC, DR>;
+  if constexpr (kX2Fits)
+    if (x2) kern = mla_append_tc_kernel_x2<DC, DR>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);

@@ -570,6 +570,39 @@ def test_cluster_and_per_tile_append_forms_agree():
     assert_close(k1.numpy()[rows], oc.kr[0], what="cluster-form k_rope")
 
 
+def test_two_ctas_per_sm_append_form_is_bit_identical():
+    """At batch 4 the Wan chunk's 148 token tiles fill one wave, one CTA per
+    SM; at batch 5 (185 tiles) two CTAs share each SM with fewer pipeline
+    stages. Both run the same MMAs in the same K order, so the four batch
+    elements they share come out bit-identical (ragged last tile included);
+    the fifth is checked against the oracle on sampled tokens."""
+    w4 = synth.workload("wan", batch=4)
+    w5 = w4.with_(batch=5)
+    weights = {k: v.cuda() for k, v in synth.draw_layer_weights(w4, 72).items()}
+    x5 = synth.draw_tokens(w5, w5.chunk_tokens, 73)
+    out = []
+    for w, x in ((w4, x5[:4]), (w5, x5)):
+        cache = V.LatentCache(V.make_config(w))
+        V.mla_cache_reset(cache)
+        pos = synth.grid_positions(w, 0, w.chunk_frames).cuda()
+        V.mla_cache_append(cache, x.contiguous().cuda(), weights["w_dkv"], weights["gamma_kv"],
+                           weights["w_kr"], pos, 0, w.chunk_frames)
+        torch.cuda.synchronize()
+        n = w.chunk_tokens
+        out.append((cache.c[:, :n].cpu(), cache.kr[:, :n].cpu()))
+    (c4, k4), (c5, k5) = out
+    assert torch.equal(c4, c5[:4]) and torch.equal(k4, k5[:4])
+    rows = np.concatenate([np.random.default_rng(3).choice(w4.chunk_tokens - 72, 20, replace=False),
+                           w4.chunk_tokens - 1 - np.arange(4)])  # + the ragged tile's last rows
+    xs = f64(x5)[4, rows]
+    pos = synth.grid_positions(w4, 0, w4.chunk_frames)[0, rows].numpy()
+    oc = O.OracleCache(1, len(rows), 1, w4.d_c, w4.d_r)
+    O.cache_append(oc, xs[None], f64(weights["w_dkv"].cpu()), f64(weights["w_kr"].cpu()), pos[None],
+                   0, 1, gamma=f64(weights["gamma_kv"].cpu()), eps=w4.rms_eps, spec=spec_of(w4))
+    assert_close(f64(c5[4, rows]), oc.c[0], what="two-per-SM form c")
+    assert_close(f64(k5[4, rows]), oc.kr[0], what="two-per-SM form k_rope")
+
+
 # ------------------------------------------------------------ error paths
 def test_position_out_of_table_sets_device_status():
     w = small()
