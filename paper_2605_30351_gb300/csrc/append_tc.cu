@@ -76,10 +76,9 @@ struct AppendShape {
   static constexpr int kStages = kFit > 6 ? 6 : kFit;
   static constexpr int kSmemBytes = 1024 + kRedOff + kStages * kStageBytes + kBarBytes + kGammaBytes;
   static constexpr uint32_t kTmemCols = N <= 32 ? 32 : (N <= 64 ? 64 : (N <= 256 ? 256 : 512));
-  // output staging row: N bf16 plus 16 bytes, so rows start on different banks
-  static constexpr int kOutStride = N * 2 + 16;
-  static_assert(kBM * kOutStride + kBM * 8 <= kStages * kStageBytes, "staging fits in the ring");
-  static_assert(kOutStride % 16 == 0 && (NC * 2) % 16 == 0, "bulk copies need 16-byte rows");
+  // output staging: dense c rows, dense k^R rows, then the rows' slots
+  static_assert(kBM * N * 2 + kBM * 8 + 16 <= kStages * kStageBytes, "staging fits in the ring");
+  static_assert(NC % 64 == 0 && (NK == 0 || NK == 32 || NK == 64), "staged row segments");
   static_assert(DC % 32 == 0 && DR % 32 == 0 && DR <= 64 && (DC <= 256 || DC % 256 == 0),
                 "shape");
   static_assert(N > 0 && NC % 32 == 0 && (NK == 0 || NK == DR), "parts");
@@ -104,6 +103,35 @@ struct AppendKParams {
   float eps;
   int* status;
 };
+
+// Writes one staged row of NCH 16-byte chunks (d holds them in order) so that
+// the eight threads of a quarter warp, which hold eight consecutive rows,
+// reach eight different bank groups: step j writes chunk j ^ m, m taken from
+// the row index (rows of 64 bytes: m = (r >> 1) & 3; of 128-byte multiples:
+// m = r & 7). A butterfly of conditional swaps puts chunk j ^ m into d[j]
+// first, so every register index stays static. The chunks land in order;
+// only the order of the writes differs between threads.
+template <int NCH>
+__device__ __forceinline__ void stage_row(uint8_t* dst, uint32_t (&d)[NCH * 4], int m) {
+#pragma unroll
+  for (int bit = 1; bit < NCH; bit <<= 1) {
+    const bool sw = (m & bit) != 0;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j)
+      if (!(j & bit)) {
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const uint32_t a = d[4 * j + w], c = d[4 * (j ^ bit) + w];
+          d[4 * j + w] = sw ? c : a;
+          d[4 * (j ^ bit) + w] = sw ? a : c;
+        }
+      }
+  }
+#pragma unroll
+  for (int j = 0; j < NCH; ++j)
+    *reinterpret_cast<uint4*>(dst + (j ^ m) * 16) =
+        make_uint4(d[4 * j], d[4 * j + 1], d[4 * j + 2], d[4 * j + 3]);
+}
 
 // tile: the token tile (128 tokens) of this CTA; c0: its first column of c
 template <int DC, int DR, int NC, int NK, int CL, int BUDGET = kSmemOne>
@@ -259,6 +287,13 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     const long long slot_n = frame_base_slot(f, p.T, p.W, p.S) + n % p.T;
     const long long my_slot =
         row_ok && debug_in_range(slot_n, 0, p.slots, p.status) ? slot_n : -1;
+    // does this row start a run of consecutive slots (row n - 1 not in the
+    // slot just below)? the tile's first row always does
+    bool run_start = my_slot >= 0 && r == 0;
+    if (my_slot >= 0 && r > 0) {
+      const long long f1 = p.first_frame + (n - 1) / p.T;
+      run_start = frame_base_slot(f1, p.T, p.W, p.S) + (n - 1) % p.T != my_slot - 1;
+    }
     float2 cs[NK > 0 ? NK / 2 : 1];
     if constexpr (NK > 0) {
       int pa[3] = {0, 0, 0};
@@ -284,15 +319,19 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
     asm volatile("bar.sync 1, 128;" ::: "memory");  // gamma_s is complete
     const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
     // Each thread stages its finished bf16 row in shared memory (the stage
-    // ring is free once the accumulator is complete). One CTA per tile then
-    // hands each row to the bulk-copy engine, one copy for its c columns and
-    // one for k^R: at the Wan shape ~1.9 us per tile, against ~2.9 us for
-    // per-thread 16-byte stores of whole rows and ~3.4 us for a coalesced
-    // store loop of the four warps after a barrier. A cluster's CTAs hold
-    // 64-column slices, whose 128-byte rows the coalesced loop writes faster
-    // than 256 small copies.
-    uint8_t* stage_out = smem;                                                     // [128][kOutStride]
-    long long* slot_of = reinterpret_cast<long long*>(smem + kBM * S::kOutStride);  // [128], clusters
+    // ring is free once the accumulator is complete): c rows dense at
+    // stage_c ([128][NC] bf16), k^R rows dense at stage_k ([128][NK]), so that
+    // a run of consecutive slots is one contiguous block in shared memory, as
+    // it is in the cache. One CTA per tile then hands each run to the
+    // bulk-copy engine (one copy for c, one for k^R, one or two runs per
+    // tile); a cluster's 64-column slices are written by a coalesced store
+    // loop, their rows not being contiguous in the cache.
+    uint8_t* stage_c = smem;
+    uint8_t* stage_k = smem + kBM * NC * 2;
+    long long* slot_of = reinterpret_cast<long long*>(smem + kBM * S::N * 2);  // [128]
+    // rows that do not continue a run (run starts and rows past the tokens),
+    // one bit per row, one word per warp
+    uint32_t* run_breaks = reinterpret_cast<uint32_t*>(slot_of + kBM);  // [4]
     // pass 1: sum of squares of this CTA's c columns (fp32)
     float ss = 0.f;
     if (have_acc) {
@@ -321,84 +360,90 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
       ss = 0.f;
       for (int q = 0; q < CL; ++q) ss += ss_all[q * kBM + r];
     }
+    const uint32_t breaks = __ballot_sync(0xffffffffu, my_slot < 0 || run_start);
     if (have_acc) {
-      const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
-      if constexpr (CL > 1) slot_of[r] = my_slot;
-      uint8_t* srow = stage_out + r * S::kOutStride;
-      // pass 2: gamma * c / rms -> bf16
-#pragma unroll 1
-      for (int cb = 0; cb < NC / 32; ++cb) {
-        uint32_t v[32];
-        tmem_ld32(t_row + cb * 32, v);
-        tmem_wait_ld();
-        uint32_t gw[16];
+      slot_of[r] = my_slot;
+      if (lane == 0) run_breaks[quarter] = breaks;
+      // positional key first, so that its RoPE factors leave the registers
+      // before pass 2: RoPE3D at the token's (t, h, w), or unrotated
+      if constexpr (NK > 0) {
+        uint32_t pk[NK / 2];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const uint4 g4 = gamma_s[cb * 4 + i];
-          gw[4 * i] = g4.x; gw[4 * i + 1] = g4.y; gw[4 * i + 2] = g4.z; gw[4 * i + 3] = g4.w;
+        for (int cb = 0; cb < NK / 32; ++cb) {
+          uint32_t v[32];
+          tmem_ld32(t_row + NC + cb * 32, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float2 f2 = cs[cb * 16 + i];
+            const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
+            pk[cb * 16 + i] = p.rotate ? pack_bf16x2(x0 * f2.x - x1 * f2.y, x0 * f2.y + x1 * f2.x)
+                                       : pack_bf16x2(x0, x1);
+          }
         }
-        uint32_t pk[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i)
-          pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]) * inv * bf16_lo(gw[i]),
-                              __uint_as_float(v[2 * i + 1]) * inv * bf16_hi(gw[i]));
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          *reinterpret_cast<uint4*>(srow + cb * 64 + i * 16) =
-              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        stage_row<NK / 8>(stage_k + r * NK * 2, pk, NK == 32 ? (r >> 1) & 3 : r & 7);
       }
-      // positional key: RoPE3D at the token's (t, h, w), or unrotated
-#pragma unroll
-      for (int cb = 0; cb < NK / 32; ++cb) {
-        uint32_t v[32];
-        tmem_ld32(t_row + NC + cb * 32, v);
+      // pass 2: gamma * c / rms -> bf16, one 64-column (128-byte) segment at a time
+      const float inv = p.use_rmsnorm ? rsqrtf(ss / DC + p.eps) : 1.f;
+      const uint32_t* gamma2 = reinterpret_cast<const uint32_t*>(gamma_s);  // bf16 pairs
+#pragma unroll 1
+      for (int sg = 0; sg < NC / 64; ++sg) {
+        uint32_t va[32], vb[32];
+        tmem_ld32(t_row + sg * 64, va);
+        tmem_ld32(t_row + sg * 64 + 32, vb);
         tmem_wait_ld();
-        uint32_t pk[16];
+        uint32_t pk[32];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const float2 f2 = cs[cb * 16 + i];
-          const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
-          pk[i] = p.rotate ? pack_bf16x2(x0 * f2.x - x1 * f2.y, x0 * f2.y + x1 * f2.x)
-                           : pack_bf16x2(x0, x1);
+          const uint32_t ga = gamma2[sg * 32 + i], gb = gamma2[sg * 32 + 16 + i];
+          pk[i] = pack_bf16x2(__uint_as_float(va[2 * i]) * inv * bf16_lo(ga),
+                              __uint_as_float(va[2 * i + 1]) * inv * bf16_hi(ga));
+          pk[16 + i] = pack_bf16x2(__uint_as_float(vb[2 * i]) * inv * bf16_lo(gb),
+                                   __uint_as_float(vb[2 * i + 1]) * inv * bf16_hi(gb));
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          *reinterpret_cast<uint4*>(srow + NC * 2 + cb * 64 + i * 16) =
-              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        stage_row<8>(stage_c + r * NC * 2 + sg * 128, pk, r & 7);
       }
     }
-    if constexpr (CL == 1) {
-      if (have_acc && my_slot >= 0) {
-        // the row's slot: c at (b * slots + slot) * d_c + c0, k^R at
-        // (b * slots + slot) * d_r; both 16-byte aligned (d_c, d_r, c0 are
-        // multiples of 32), as is the staged row (kOutStride is)
-        const uint8_t* srow = stage_out + r * S::kOutStride;
-        const size_t row_id = static_cast<size_t>(b) * p.slots + my_slot;
-        fence_proxy_async_smem();
-        if constexpr (NC > 0) bulk_store(p.c + row_id * DC + c0, srow, NC * 2);
-        if constexpr (NK > 0) bulk_store(p.kr + row_id * DR, srow + NC * 2, NK * 2);
-        bulk_commit();
-        bulk_wait_read_all();  // the staging rows must outlive the copies' reads
-      }
-    } else {
-      // the four epilogue warps only: consecutive threads store consecutive
-      // 16-byte pieces of the staged rows
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (have_acc) {
+    // the staged rows reach the async proxy (the bulk copies), then the four
+    // epilogue warps meet; a wait that gave up anywhere shows in abort_flag
+    fence_proxy_async_smem();
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (have_acc && !*abort_flag) {
+      if constexpr (CL == 1) {
+        // the thread whose row starts a run of consecutive slots copies the
+        // run: c rows to (b * slots + slot) * d_c (+ c0), k^R rows to
+        // (b * slots + slot) * d_r, all 16-byte aligned and sized
+        if (run_start) {
+          int end = kBM;  // the next row that does not continue this run
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            uint32_t m = w < quarter ? 0u : run_breaks[w];
+            if (w == quarter) m &= ~((2u << lane) - 1u);  // rows after this one
+            if (m != 0u && end == kBM) end = w * 32 + __ffs(static_cast<int>(m)) - 1;
+          }
+          const int len = end - r;
+          const size_t row_id = static_cast<size_t>(b) * p.slots + my_slot;
+          if constexpr (NC > 0)
+            bulk_store(p.c + row_id * DC + c0, stage_c + r * NC * 2, len * NC * 2);
+          if constexpr (NK > 0) bulk_store(p.kr + row_id * DR, stage_k + r * NK * 2, len * NK * 2);
+          bulk_commit();
+          bulk_wait_read_all();  // the staged rows must outlive the copies' reads
+        }
+      } else {
+        // consecutive threads store consecutive 16-byte pieces of the rows
         constexpr int kChunks = S::N * 2 / 16;  // 16-byte pieces per output row
         constexpr int kChunksC = NC * 2 / 16;
         for (int q = r; q < kBM * kChunks; q += kBM) {
           const int row = q / kChunks, ch = q % kChunks;
           const long long slot = slot_of[row];
           if (slot < 0) continue;
-          const uint4 v =
-              *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
+          const size_t row_id = static_cast<size_t>(b) * p.slots + slot;
           if (ch < kChunksC)
-            *reinterpret_cast<uint4*>(p.c + (static_cast<size_t>(b) * p.slots + slot) * DC +
-                                      c0 + ch * 8) = v;
+            *reinterpret_cast<uint4*>(p.c + row_id * DC + c0 + ch * 8) =
+                *reinterpret_cast<const uint4*>(stage_c + row * NC * 2 + ch * 16);
           else
-            *reinterpret_cast<uint4*>(p.kr + (static_cast<size_t>(b) * p.slots + slot) * DR +
-                                      (ch - kChunksC) * 8) = v;
+            *reinterpret_cast<uint4*>(p.kr + row_id * DR + (ch - kChunksC) * 8) =
+                *reinterpret_cast<const uint4*>(stage_k + row * NK * 2 + (ch - kChunksC) * 16);
         }
       }
     }
