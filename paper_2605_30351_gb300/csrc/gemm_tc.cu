@@ -8,7 +8,8 @@
 //   warp 1     TMEM allocation; one lane issues tcgen05.mma (N = BN, or two
 //              MMAs of N = BN/2 when BN > 256)
 //   warps 2-5  epilogue, thread i = row i: TMEM -> registers -> bf16 staged
-//              in shared memory, then stored by all 128 threads together.
+//              in shared memory, then one bulk copy per row (two when the row
+//              straddles kRowScale's split between C and C2).
 // Epilogues:
 //   kStore      plain bf16 C
 //   kStoreSq    bf16 C plus, per row, the sum of squares of this tile's fp32
@@ -46,7 +47,6 @@ struct GemmShape {
   static constexpr int kFit = (232448 - 1024 - kBarBytes) / kStageBytes;
   static constexpr int kStages = kFit > MAXST ? MAXST : kFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
-  static constexpr int kOutStride = BN * 2 + 16;  // staged bf16 row + 16 bytes (bank spread)
   static constexpr uint32_t kTmemCols = BN <= 128 ? 128 : (BN <= 256 ? 256 : 512);
   static constexpr int kHalves = BN > 256 ? 2 : 1;  // MMAs (and B boxes) per K step
   static constexpr int kBN1 = BN / kHalves;         // columns of one MMA
@@ -55,7 +55,8 @@ struct GemmShape {
   static_assert(!PAIR || (BN <= 256 && BN % 32 == 0), "paired MMA: one N <= 256 MMA, 16-row B halves");
   static_assert(BN % 32 == 0 && BN <= 512 && kBN1 % 32 == 0, "tile width");
   static_assert(kStageBytes % 1024 == 0, "swizzle-atom alignment");
-  static_assert(kBM * kOutStride <= kStages * kStageBytes, "staging fits in the ring");
+  static_assert(kBM * BN * 2 <= kStages * kStageBytes, "staging fits in the ring");
+  static_assert(BN % 64 == 0, "rows staged in 64-column segments");
 };
 
 struct GemmKParams {
@@ -200,57 +201,62 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = quarter * 32 + lane;
     const uint32_t t_row = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int m = m0 + r;
-    const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
-    uint8_t* stage_out = smem;  // [128][kOutStride]
     const int n_valid = min(BN, p.N - n0);
+    // kRowScale: the row's statistics (written by the previous GEMM) are
+    // fetched while the MMAs run, so no global load follows the accumulator
+    float scale = 1.f;
+    if constexpr (EPI == kRowScale) {
+      float ss = 0.f;
+      if (m < p.M)
+        for (int t = 0; t < p.sq_tiles; ++t) ss += p.sq[static_cast<size_t>(t) * p.M + m];
+      scale = rsqrtf(ss / p.sq_dim + p.eps);
+    }
+    const bool have_acc = mbar_wait(acc_full, 0, wc) && !*abort_flag;
+    // Each thread stages its row densely in shared memory ([128][BN] bf16,
+    // the ring being free once the accumulator is complete; chunk order
+    // rotated per row so the quarter warp's rows hit distinct banks) and
+    // hands it to the bulk-copy engine, one copy per destination matrix.
+    uint8_t* srow = smem + r * BN * 2;
     if (have_acc) {
       tc_fence_after();
-      float scale = 1.f;
-      if constexpr (EPI == kRowScale) {
-        float ss = 0.f;
-        if (m < p.M)
-          for (int t = 0; t < p.sq_tiles; ++t) ss += p.sq[static_cast<size_t>(t) * p.M + m];
-        scale = rsqrtf(ss / p.sq_dim + p.eps);
-      }
       float ss_own = 0.f;
-      uint8_t* srow = stage_out + r * S::kOutStride;
 #pragma unroll 1
-      for (int cb = 0; cb < BN / 32; ++cb) {
-        uint32_t v[32];
-        tmem_ld32(t_row + cb * 32, v);
+      for (int sg = 0; sg < BN / 64; ++sg) {
+        uint32_t va[32], vb[32];
+        tmem_ld32(t_row + sg * 64, va);
+        tmem_ld32(t_row + sg * 64 + 32, vb);
         tmem_wait_ld();
-        uint32_t pk[16];
+        uint32_t pk[32];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float a0 = __uint_as_float(v[2 * i]), a1 = __uint_as_float(v[2 * i + 1]);
+        for (int i = 0; i < 32; ++i) {
+          const uint32_t* v = i < 16 ? va : vb;
+          const int j = i & 15;
+          const float a0 = __uint_as_float(v[2 * j]), a1 = __uint_as_float(v[2 * j + 1]);
           if constexpr (EPI == kStoreSq) {
-            const int col = cb * 32 + 2 * i;
+            const int col = sg * 64 + 2 * i;
             if (col < n_valid) ss_own = fmaf(a0, a0, ss_own);
             if (col + 1 < n_valid) ss_own = fmaf(a1, a1, ss_own);
           }
           pk[i] = pack_bf16x2(a0 * scale, a1 * scale);
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          *reinterpret_cast<uint4*>(srow + cb * 64 + i * 16) =
-              make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        stage_row<8>(srow + sg * 128, pk, r & 7);
       }
       if constexpr (EPI == kStoreSq)
         if (m < p.M) p.sq[static_cast<size_t>(n_tile) * p.M + m] = ss_own;
-    }
-    asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
-    if (have_acc) {
-      const int chunks = n_valid / 8;  // 16-byte pieces per row (N is a multiple of 8)
-      for (int q = r; q < kBM * chunks; q += kBM) {
-        const int row = q / chunks, ch = q % chunks;
-        const int mm = m0 + row;
-        if (mm >= p.M) continue;
-        const uint4 v = *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
-        const int col = n0 + ch * 8;
-        if (EPI == kRowScale && col >= p.split)
-          *reinterpret_cast<uint4*>(p.c2 + static_cast<size_t>(mm) * p.ld2 + (col - p.split)) = v;
-        else
-          *reinterpret_cast<uint4*>(p.c + static_cast<size_t>(mm) * p.ldc + col) = v;
+      if (m < p.M) {
+        // columns [n0, n0 + n_valid) of row m: below `split` to C, from it to
+        // C2; addresses and sizes are multiples of 16 bytes (N, split, the
+        // leading dimensions and n0 are multiples of 8)
+        int c_end = n_valid;
+        if constexpr (EPI == kRowScale) c_end = max(0, min(n_valid, p.split - n0));
+        fence_proxy_async_smem();
+        if (c_end > 0) bulk_store(p.c + static_cast<size_t>(m) * p.ldc + n0, srow, c_end * 2);
+        if constexpr (EPI == kRowScale)
+          if (c_end < n_valid)
+            bulk_store(p.c2 + static_cast<size_t>(m) * p.ld2 + (n0 + c_end - p.split),
+                       srow + c_end * 2, (n_valid - c_end) * 2);
+        bulk_commit();
+        bulk_wait_read_all();  // the staged row must outlive the copies' reads
       }
     }
   }

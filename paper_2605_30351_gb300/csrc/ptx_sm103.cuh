@@ -194,6 +194,35 @@ __device__ __forceinline__ void bulk_wait_read_all() {
   asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
+// Writes one staged row of NCH 16-byte chunks (d holds them in order) so that
+// the eight threads of a quarter warp, which hold eight consecutive rows,
+// reach eight different bank groups: step j writes chunk j ^ m, m taken from
+// the row index (rows of 64 bytes: m = (r >> 1) & 3; of 128-byte multiples:
+// m = r & 7). A butterfly of conditional swaps puts chunk j ^ m into d[j]
+// first, so every register index stays static. The chunks land in order;
+// only the order of the writes differs between threads.
+template <int NCH>
+__device__ __forceinline__ void stage_row(uint8_t* dst, uint32_t (&d)[NCH * 4], int m) {
+#pragma unroll
+  for (int bit = 1; bit < NCH; bit <<= 1) {
+    const bool sw = (m & bit) != 0;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j)
+      if (!(j & bit)) {
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const uint32_t a = d[4 * j + w], c = d[4 * (j ^ bit) + w];
+          d[4 * j + w] = sw ? c : a;
+          d[4 * (j ^ bit) + w] = sw ? a : c;
+        }
+      }
+  }
+#pragma unroll
+  for (int j = 0; j < NCH; ++j)
+    *reinterpret_cast<uint4*>(dst + (j ^ m) * 16) =
+        make_uint4(d[4 * j], d[4 * j + 1], d[4 * j + 2], d[4 * j + 3]);
+}
+
 // ------------------------------------------------------------------ tcgen05
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {  // whole warp
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
