@@ -494,27 +494,48 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_arrive(p_full);
     }
 
-    if (ok && mbar_wait(pv_done, (nblk - 1) & 1, wc)) {
+    // O / l as bf16: each thread stages its row densely in the key stages
+    // (free once the last PV is done: every key tile, the peer's multicast
+    // halves included, has landed and been read) and the rows leave shared
+    // memory by bulk copy, the whole tile at once when its rows are
+    // consecutive rows of o (DV = d_c).
+    const bool have_o = ok && mbar_wait(pv_done, (nblk - 1) & 1, wc);
+    uint8_t* srow = sKV + r * DV * 2;
+    if (have_o) {
       tc_fence_after();
       const float inv_l = 1.f / l_run;
-      uint4* dst = reinterpret_cast<uint4*>(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC +
-                                            vpart * DV);
 #pragma unroll 1
-      for (int c = 0; c < DV / 32; ++c) {
-        uint32_t ov[32];
-        tmem_ld32(tmem + t_lane + S::kTmemO + c * 32, ov);
+      for (int sg = 0; sg < DV / 64; ++sg) {
+        uint32_t va[32], vb[32];
+        tmem_ld32(tmem + t_lane + S::kTmemO + sg * 64, va);
+        tmem_ld32(tmem + t_lane + S::kTmemO + sg * 64 + 32, vb);
         tmem_wait_ld();
-        uint32_t pk[16];
+        uint32_t pk[32];
 #pragma unroll
-        for (int i = 0; i < 16; ++i)
-          pk[i] = pack_bf16x2(__uint_as_float(ov[2 * i]) * inv_l,
-                              __uint_as_float(ov[2 * i + 1]) * inv_l);
-        if (row_ok) {
-#pragma unroll
-          for (int i = 0; i < 4; ++i)
-            dst[c * 4 + i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        for (int i = 0; i < 32; ++i) {
+          const uint32_t* v = i < 16 ? va : vb;
+          const int j = i & 15;
+          pk[i] = pack_bf16x2(__uint_as_float(v[2 * j]) * inv_l,
+                              __uint_as_float(v[2 * j + 1]) * inv_l);
         }
+        stage_row<8>(srow + sg * 128, pk, r & 7);
       }
+    }
+    fence_proxy_async_smem();
+    if constexpr (DV == DC) {
+      asm volatile("bar.sync 1, 128;" ::: "memory");  // the four softmax warps
+      // the tile's rows below p.rows; none in the CTA that only pads the grid
+      // to whole clusters (an odd number of row tiles)
+      const int valid = min(kBM, p.rows - row0);
+      if (r == 0 && have_o && !*abort_flag && valid > 0) {
+        bulk_store(p.o + (static_cast<size_t>(b) * p.rows + row0) * DC, sKV, valid * DC * 2);
+        bulk_commit();
+        bulk_wait_read_all();  // the staged rows must outlive the copy's reads
+      }
+    } else if (have_o && row_ok) {
+      bulk_store(p.o + (static_cast<size_t>(b) * p.rows + grow) * DC + vpart * DV, srow, DV * 2);
+      bulk_commit();
+      bulk_wait_read_all();
     }
   }
 
