@@ -275,6 +275,296 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Persistent paired-SM form, for large M. One CTA per SM; each cluster of
+// two (an SM pair) walks the pair tiles t = cluster, cluster + clusters, ...
+// (a pair tile: M tiles 2i and 2i + 1 of one N tile, N tiles fastest, so the
+// pairs working at one moment share their A rows in L2). The stage ring runs
+// on across tile boundaries, and two TMEM accumulators of BN columns let the
+// epilogue warps drain one tile while the MMAs fill the next; a non-
+// persistent CTA instead pays its set-up, pipeline fill and epilogue once
+// per tile. The staged output rows have their own shared memory, apart from
+// the ring.
+template <int BN>
+struct PGemmShape {
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBox = BN / 2;  // B rows per CTA
+  static constexpr int kBBytes = kBBox * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kTxBytes = 2 * kStageBytes;  // the even CTA's full barrier counts both
+  static constexpr int kStagingBytes = kBM * BN * 2;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kFit = (232448 - 1024 - kBarBytes - kStagingBytes) / kStageBytes;
+  static constexpr int kStages = kFit > 8 ? 8 : kFit;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kStagingBytes + kBarBytes;
+  static constexpr uint32_t kAccStride = 256;  // TMEM columns per accumulator
+  static constexpr uint32_t kTmemCols = 512;
+  static constexpr uint32_t kIdesc = idesc_bf16_f32(2 * kBM, BN, false, false);
+  static_assert(BN % 64 == 0 && BN <= 256, "one N <= 256 MMA, rows staged in 64-column segments");
+  static_assert(kStages >= 3, "ring depth");
+  static_assert(kStageBytes % 1024 == 0 && kStagingBytes % 1024 == 0, "swizzle-atom alignment");
+  static_assert(2 * kStages + 5 <= kBarBytes / 8 - 1, "barriers, TMEM slot and abort flag");
+};
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_gemm_tc_persistent_kernel(const __grid_constant__ CUtensorMap tm_a,
+                                  const __grid_constant__ CUtensorMap tm_b, const GemmKParams p) {
+  using S = PGemmShape<BN>;
+  constexpr int NST = S::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align_smem_1024(smem_raw);
+  uint8_t* staging = smem + NST * S::kStageBytes;  // [128][BN] bf16
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + S::kStagingBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + NST;
+  uint64_t* acc_full = bars + 2 * NST;  // [2]
+  uint64_t* acc_empty = acc_full + 2;   // [2], used in the even CTA
+  uint64_t* mma_drain = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int cluster = blockIdx.x / 2;
+  const int clusters = gridDim.x / 2;
+  const int n_tiles = (p.N + BN - 1) / BN;
+  const int m_pairs = ((p.M + kBM - 1) / kBM + 1) / 2;
+  const int total = n_tiles * m_pairs;
+  const int k_blocks = p.K / kBK;
+  const WaitCtx wc{abort_flag, p.status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 2 * 128);  // every epilogue thread of both CTAs
+    }
+    mbar_init(mma_drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, S::kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int crank = static_cast<int>(cluster_ctarank());
+  cluster_sync();  // the peer's barriers exist before copies, commits and arrivals reach them
+  grid_dep_sync();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_a);
+      tma_prefetch_desc(&tm_b);
+      int it = 0;  // k blocks issued so far, over all tiles
+      bool ok = true;
+      for (int t = cluster; t < total && ok; t += clusters) {
+        const int n0 = (t % n_tiles) * BN;
+        const int m0 = (2 * (t / n_tiles) + crank) * kBM;
+        for (int kb = 0; kb < k_blocks; ++kb) {
+          const int st = it % NST;
+          if (it >= NST && !mbar_wait(&empty[st], ((it / NST) - 1) & 1, wc)) {
+            ok = false;
+            break;
+          }
+          uint8_t* a = smem + st * S::kStageBytes;
+          const uint32_t bar = dsmem_addr(smem_u32(&full[st]), 0);
+          if (crank == 0) mbar_arrive_expect_tx(&full[st], S::kTxBytes);
+          tma_load_2d_pair(a, &tm_a, bar, kb * kBK, m0);
+          tma_load_2d_pair(a + S::kABytes, &tm_b, bar, kb * kBK, n0 + crank * S::kBBox);
+          ++it;
+        }
+      }
+      // the even CTA's MMAs release this CTA's stages: the last releases must
+      // have landed before the CTA may exit
+      for (int u = it > NST ? it - NST : 0; u < it && !*abort_flag; ++u)
+        mbar_wait(&empty[u % NST], (u / NST) & 1, wc);
+      if (*abort_flag && crank == 0)
+        for (int u = it > NST ? it - NST : 0; u < it; ++u)
+          mbar_wait_drain(&full[u % NST], (u / NST) & 1, p.status);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && crank == 0) {
+      int it = 0, tl = 0;
+      bool ok = true;
+      for (int t = cluster; t < total && ok; t += clusters, ++tl) {
+        const int buf = tl & 1;
+        // both CTAs' epilogues have drained this accumulator (two tiles ago)
+        if (tl >= 2 && !mbar_wait_cluster(&acc_empty[buf], ((tl >> 1) - 1) & 1, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc = tmem + buf * S::kAccStride;
+        for (int kb = 0; kb < k_blocks; ++kb, ++it) {
+          const int st = it % NST;
+          if (!mbar_wait(&full[st], (it / NST) & 1, wc)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t aa = smem_u32(smem + st * S::kStageBytes);
+          const uint32_t ba = aa + S::kABytes;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            umma_pair_ss(acc, sdesc(aa + k * 32, 16, 1024, kSw128),
+                         sdesc(ba + k * 32, 16, 1024, kSw128), S::kIdesc, (kb | k) != 0 ? 1u : 0u);
+          umma_pair_commit_mc(&empty[st], 3);
+        }
+        if (ok) umma_pair_commit_mc(&acc_full[buf], 3);
+      }
+      if (!ok) {  // every MMA issued must be done before the CTA moves on
+        umma_pair_commit_mc(mma_drain, 1);
+        mbar_wait_drain(mma_drain, 0, p.status);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t t_lane = static_cast<uint32_t>(quarter * 32) << 16;
+    uint8_t* srow = staging + r * BN * 2;
+    int tl = 0;
+    for (int t = cluster; t < total; t += clusters, ++tl) {
+      const int buf = tl & 1;
+      const int n_tile = t % n_tiles;
+      const int n0 = n_tile * BN;
+      const int m = (2 * (t / n_tiles) + crank) * kBM + r;
+      const int n_valid = min(BN, p.N - n0);
+      // kRowScale: the row's statistics (from the previous GEMM), fetched
+      // before the accumulator is ready
+      float scale = 1.f;
+      if constexpr (EPI == kRowScale) {
+        float ss = 0.f;
+        if (m < p.M)
+          for (int q = 0; q < p.sq_tiles; ++q) ss += p.sq[static_cast<size_t>(q) * p.M + m];
+        scale = rsqrtf(ss / p.sq_dim + p.eps);
+      }
+      if (!mbar_wait(&acc_full[buf], (tl >> 1) & 1, wc)) break;
+      tc_fence_after();
+      bulk_wait_read_all();  // the previous tile's copy of this row has read it
+      float ss_own = 0.f;
+      const uint32_t acc = tmem + t_lane + buf * S::kAccStride;
+#pragma unroll 1
+      for (int sg = 0; sg < BN / 64; ++sg) {
+        uint32_t va[32], vb[32];
+        tmem_ld32(acc + sg * 64, va);
+        tmem_ld32(acc + sg * 64 + 32, vb);
+        tmem_wait_ld();
+        uint32_t pk[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const uint32_t* v = i < 16 ? va : vb;
+          const int j = i & 15;
+          const float a0 = __uint_as_float(v[2 * j]), a1 = __uint_as_float(v[2 * j + 1]);
+          if constexpr (EPI == kStoreSq) {
+            const int col = sg * 64 + 2 * i;
+            if (col < n_valid) ss_own = fmaf(a0, a0, ss_own);
+            if (col + 1 < n_valid) ss_own = fmaf(a1, a1, ss_own);
+          }
+          pk[i] = pack_bf16x2(a0 * scale, a1 * scale);
+        }
+        stage_row<8>(srow + sg * 128, pk, r & 7);
+      }
+      // this thread's reads of the accumulator are done: release it to the
+      // MMA issuer (in the even CTA)
+      tc_fence_before();
+      mbar_arrive_cluster(dsmem_addr(smem_u32(&acc_empty[buf]), 0));
+      if constexpr (EPI == kStoreSq)
+        if (m < p.M) p.sq[static_cast<size_t>(n_tile) * p.M + m] = ss_own;
+      if (m < p.M) {
+        // columns [n0, n0 + n_valid) of row m: below `split` to C, from it to
+        // C2 (16-byte aligned and sized, as in the non-persistent form)
+        int c_end = n_valid;
+        if constexpr (EPI == kRowScale) c_end = max(0, min(n_valid, p.split - n0));
+        fence_proxy_async_smem();
+        if (c_end > 0) bulk_store(p.c + static_cast<size_t>(m) * p.ldc + n0, srow, c_end * 2);
+        if constexpr (EPI == kRowScale)
+          if (c_end < n_valid)
+            bulk_store(p.c2 + static_cast<size_t>(m) * p.ld2 + (n0 + c_end - p.split),
+                       srow + c_end * 2, (n_valid - c_end) * 2);
+        bulk_commit();
+      }
+    }
+    bulk_wait_read_all();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs are done with the pair's TMEM and barriers
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, S::kTmemCols);
+  }
+}
+
+template <int BN, int EPI>
+int launch_gemm_persistent(const void* a, const void* b, int M, int N, int K, GemmKParams kp,
+                           cudaStream_t stream) {
+  using S = PGemmShape<BN>;
+  if (K % kBK != 0 || N % 8 != 0) return MLA_ERR_UNSUPPORTED;
+  CUtensorMap tm_a, tm_b;
+  if (!encode_map_2d_bf16(&tm_a, a, K, M, K * 2ull, kBK, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_2d_bf16(&tm_b, b, K, N, K * 2ull, kBK, S::kBBox, CU_TENSOR_MAP_SWIZZLE_128B))
+    return MLA_ERR_CUDA;
+  auto kern = mla_gemm_tc_persistent_kernel<BN, EPI>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmemBytes);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  kp.M = M;
+  kp.N = N;
+  kp.K = K;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = S::kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see grid_dep_sync
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  // as many clusters as are resident at once (one CTA per SM), at most one
+  // per pair tile
+  static int resident = -1;  // per process, for this instantiation
+  if (resident < 0) {
+    int n = 0;
+    cudaLaunchConfig_t oc = cfg;
+    oc.gridDim = dim3(2, 1, 1);
+    oc.numAttrs = 2;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &oc) != cudaSuccess) {
+      cudaGetLastError();
+      n = 0;
+    }
+    resident = n;
+  }
+  if (resident < 1) return MLA_ERR_UNSUPPORTED;
+  const long long m_pairs = ((M + kBM - 1) / kBM + 1) / 2;
+  const long long total = m_pairs * ((N + BN - 1) / BN);
+  const int clusters = static_cast<int>(total < resident ? total : resident);
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  e = cudaLaunchKernelEx(&cfg, kern, tm_a, tm_b, kp);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return MLA_ERR_CUDA;
+  }
+  return MLA_OK;
+}
+
 template <int BN, int EPI, int MAXST = 6, bool PAIR = false>
 int launch_gemm(const void* a, const void* b, int M, int N, int K, GemmKParams kp,
                 cudaStream_t stream) {
@@ -408,8 +698,10 @@ int launch_query_prologue(const QueryArgs& a) {
   // pair of SMs (three 32 KB stages each): each SM streams half of every B
   // tile (four Wan chunks: 132.8 -> 129.3 us for both GEMMs, same outputs)
   int rc = narrow ? launch_gemm<kQuerySqTile, kStoreSq>(a.x, a.w_dq, M, a.d_q, a.hidden, k1, a.stream)
-                  : launch_gemm<256, kStoreSq, 3, true>(a.x, a.w_dq, M, a.d_q, a.hidden, k1,
-                                                        a.stream);
+                  : launch_gemm_persistent<256, kStoreSq>(a.x, a.w_dq, M, a.d_q, a.hidden, k1,
+                                                          a.stream);
+  if (rc == MLA_ERR_UNSUPPORTED && !narrow)
+    rc = launch_gemm<256, kStoreSq, 3, true>(a.x, a.w_dq, M, a.d_q, a.hidden, k1, a.stream);
   if (rc != MLA_OK) return rc;
   // [q_c | q_r] = (c~ / rms(c~)) [W_qc ; W_qr]^T with gamma folded into the weights
   GemmKParams k2 = {};
@@ -426,9 +718,13 @@ int launch_query_prologue(const QueryArgs& a) {
   // two-stage ring: two CTAs per SM overlap one tile's epilogue with the next
   // one's loads (measured 48 vs 51 us at one Wan chunk, 138 vs 164 us at four);
   // large M: the paired-SM form, as for the first GEMM
-  if (!narrow)
+  if (!narrow) {
+    rc = launch_gemm_persistent<256, kRowScale>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
+                                                a.d_q, k2, a.stream);
+    if (rc != MLA_ERR_UNSUPPORTED) return rc;
     return launch_gemm<256, kRowScale, 3, true>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
                                                 a.d_q, k2, a.stream);
+  }
   return launch_gemm<256, kRowScale, 2>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
                                         a.d_q, k2, a.stream);
 }
@@ -494,6 +790,9 @@ int launch_output_projection(const OutProjArgs& a) {
                                        a.stream);
   // large M: paired-SM MMAs (each SM streams half of every B tile; four Wan
   // chunks: 97.3 -> 85.9 us, same output)
+  const int rc = launch_gemm_persistent<256, kStore>(a.o_lat, a.w_b, a.rows, a.hidden,
+                                                     a.heads * a.d_c, k, a.stream);
+  if (rc != MLA_ERR_UNSUPPORTED) return rc;
   return launch_gemm<256, kStore, 3, true>(a.o_lat, a.w_b, a.rows, a.hidden, a.heads * a.d_c, k,
                                            a.stream);
 }
