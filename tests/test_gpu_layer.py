@@ -76,13 +76,18 @@ def test_query_prologue_matches_oracle(nq, batch, shape):
     assert_close(f64(q_r), ref_qr, what="q_r")
 
 
-def test_layer_gemms_at_four_chunks_match_oracle():
+@pytest.mark.parametrize("heads,d_c", [(12, 192), (3, 64)])
+def test_layer_gemms_at_four_chunks_match_oracle(heads, d_c):
     """Four Wan-1.3B chunks (18,720 query tokens): both query-prologue GEMMs and
-    the output projection take 256-wide tiles as paired-SM MMAs (two M tiles
-    per M = 256 MMA, each CTA holding half of the B rows; 147 M tiles, so the
-    last pair has a tile past the tokens). Sampled rows, including the first
-    and last pair, against the oracle (Eqs. cq, qnope, qrope, absorb-v)."""
-    w = synth.workload("wan", batch=4)
+    the output projection run the persistent paired-SM kernel (two M tiles per
+    M = 256 MMA, each CTA holding half of the B rows, clusters walking the
+    pair tiles; 147 M tiles, so the last pair has a tile past the tokens).
+    With 3 heads of d_c = 64 the absorbed query GEMM has N = 288: its first
+    256-wide tile straddles the q_c | q_r split at column 192 and its second
+    is ragged, and the output projection's K (192) is three K blocks, fewer
+    than the ring's stages. Sampled rows, including the first and last pair,
+    against the oracle (Eqs. cq, qnope, qrope, absorb-v)."""
+    w = synth.workload("wan", batch=4, heads=heads, d_c=d_c)
     nq = w.chunk_tokens
     wt = synth.draw_layer_weights(w, seed=74)
     dev = {k: v.cuda() for k, v in wt.items()}
