@@ -334,8 +334,8 @@ int mla_dense_attention_forward(const mla_config* cfg, const void* q, const void
  *  w_uv  bf16 [heads][head_dim][d_c]          W_up^V
  *  k, v  bf16 [batch][heads][W*T][head_dim]   outputs (caller-owned)
  * MLA_ERR_ARG for a cache with MLA_FLAG_ROTATE_AT_USE (its k is unrotated);
- * MLA_ERR_UNSUPPORTED unless d_c is a multiple of 64 and head_dim - d_r a
- * multiple of 8.
+ * MLA_ERR_UNSUPPORTED unless d_c is a multiple of 64 and head_dim and
+ * head_dim - d_r are multiples of 32.
  */
 int mla_decompress_window(const mla_cache* cache, const void* w_uk, const void* w_uv, void* k,
                           void* v, void* stream);

@@ -8,19 +8,26 @@
 // [W_up^K ; W_up^V] (H*d_nope + H*head_dim of them) cut into tiles of BN;
 // CTA (t, g) keeps column tile t of the weights in shared memory for its
 // whole life and streams the 128-slot tiles g, g + G, g + 2G, ... of c
-// through a two-stage TMA ring. Accumulators alternate between two TMEM
-// buffers, so the epilogue of one tile overlaps the MMA of the next. The
-// weights leave L2 once per CTA and c once per column tile, and every output
-// byte is written once; at the Wan window the 201 MB of keys and values
-// written dominate, so the kernel is bound by HBM writes.
+// through a two-stage TMA ring; a tile never spans two batch elements (each
+// element's slots are cut into tiles of their own, the last one ragged).
+// Accumulators alternate between two TMEM buffers, so the epilogue of one
+// tile overlaps the MMA of the next. The weights leave L2 once per CTA and c
+// once per column tile, and every output byte is written once; at the Wan
+// window the 201 MB of keys and values written dominate, so the kernel is
+// bound by HBM writes.
 //   warp 0     TMA producer (weights once, then c tiles)
 //   warp 1     TMEM allocation; one lane issues tcgen05.mma (M = 128, N = BN)
 //   warps 2-13 epilogue: warps w, w + 4, w + 8 read TMEM lane quarter w % 4
-//              (slot rows), each a third of the columns, into a shared staging
-//              tile as bf16; then all 384 threads store it with 16-byte stores
-//              into the head-major outputs. Key tiles also copy each slot's cached
-//              positional key behind every head that starts in the tile; those
-//              loads are issued before the TMEM reads so their latency hides.
+//              (slot rows), each a third of the columns, into shared staging
+//              as bf16: one [128 slots x 32 columns] box per 32 columns, in
+//              the 64-byte swizzle of the output tensor maps. One thread then
+//              writes the tile with a TMA tensor store per box (a box never
+//              spans two heads: d_nope and head_dim are multiples of 32; slots
+//              past the element's last are clipped by the map). Key tiles
+//              also copy each slot's cached positional key behind every head
+//              that starts in the tile, with 16-byte stores from registers;
+//              those loads are issued before the TMEM reads so their latency
+//              hides.
 #include "internal.h"
 #include "ptx_sm103.cuh"
 
@@ -40,18 +47,17 @@ struct DecShape {
   static constexpr int kChunkBytesW = BN * 128;   // one [BN x 64] bf16 K-chunk
   static constexpr int kWBytes = (DC / 64) * kChunkBytesW;
   static constexpr int kCBytes = (DC / 64) * kChunkBytesC;
-  static constexpr int kOutStride = BN * 2 + 16;  // staged bf16 row + 16 bytes (bank spread)
+  static constexpr int kBoxBytes = kBM * 64;  // one staged [128 slots x 32 columns] box, SW64
   static constexpr int kStageOff = kWBytes + 2 * kCBytes;
-  static constexpr int kBarOff = kStageOff + kBM * kOutStride;
-  // per-row and per-chunk output offsets, so the store loop does no division
+  static constexpr int kBarOff = kStageOff + (BN / 32) * kBoxBytes;
+  // per-row output offsets of the positional-key copies
   static constexpr int kRowTabOff = kBarOff + 128;             // long long [128]
-  static constexpr int kColTabOff = kRowTabOff + kBM * 8;      // long long [BN/8]
-  static constexpr int kHeadTabOff = kColTabOff + (BN / 8) * 8;  // long long [BN/8]
+  static constexpr int kHeadTabOff = kRowTabOff + kBM * 8;     // long long [BN/8]
   static constexpr int kSmemBytes = 1024 + kHeadTabOff + (BN / 8) * 8;
   static constexpr uint32_t kTmemCols = 2 * BN <= 256 ? 256 : 512;
   static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN, false, false);
   static_assert(DC % 64 == 0 && DC <= 256, "latent width");
-  static_assert(BN % 32 == 0 && BN % 16 == 0 && BN <= 256, "tile width");
+  static_assert(BN % 32 == 0 && BN <= 256, "tile width: whole 32-column boxes");
   static_assert(kChunkBytesW % 1024 == 0 && kStageOff % 1024 == 0, "swizzle-atom alignment");
   static_assert(kSmemBytes <= 232448, "shared memory");
 };
@@ -60,7 +66,7 @@ struct DecKParams {
   const __nv_bfloat16* kr;  // [M][d_r]
   __nv_bfloat16* k;         // [B][H][slots][head_dim]
   __nv_bfloat16* v;
-  int M, n_row_tiles, tiles_k, cols_k, cols_v, dn, head_dim, d_r, slots, heads;
+  int M, tiles_per_b, n_row_tiles, tiles_k, cols_k, cols_v, dn, head_dim, d_r, slots, heads;
   int* status;
 };
 
@@ -86,7 +92,9 @@ template <int DC>
 __global__ void __launch_bounds__(kThreads, 1)
     mla_decompress_tc_kernel(const __grid_constant__ CUtensorMap tm_c,
                              const __grid_constant__ CUtensorMap tm_wk,
-                             const __grid_constant__ CUtensorMap tm_wv, const DecKParams p) {
+                             const __grid_constant__ CUtensorMap tm_wv,
+                             const __grid_constant__ CUtensorMap tm_ko,
+                             const __grid_constant__ CUtensorMap tm_vo, const DecKParams p) {
   using S = DecShape<DC>;
   constexpr int BN = S::BN;
   constexpr int KC = DC / 64;
@@ -105,7 +113,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   long long* row_base = reinterpret_cast<long long*>(smem + S::kRowTabOff);
-  long long* col_off = reinterpret_cast<long long*>(smem + S::kColTabOff);
   long long* head_off = reinterpret_cast<long long*>(smem + S::kHeadTabOff);
 
   const int warp = threadIdx.x >> 5;
@@ -152,9 +159,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = i & 1;
         if (i >= 2 && !mbar_wait(&c_empty[s], ((i >> 1) - 1) & 1, wc)) break;
         mbar_arrive_expect_tx(&c_full[s], S::kCBytes);
+        // slots t*128 .. of batch element bb (rows past its last slot are
+        // loaded but never stored)
+        const int m0 = (r / p.tiles_per_b) * p.slots + (r % p.tiles_per_b) * kBM;
         for (int kc = 0; kc < KC; ++kc)
-          tma_load_2d(sC + s * S::kCBytes + kc * S::kChunkBytesC, &tm_c, &c_full[s], kc * 64,
-                      r * kBM);
+          tma_load_2d(sC + s * S::kCBytes + kc * S::kChunkBytesC, &tm_c, &c_full[s], kc * 64, m0);
         issued = i + 1;
       }
       if (*abort_flag) {  // let our own copies land before the CTA exits
@@ -198,18 +207,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int et = part * kBM + rl;         // index among the epilogue threads
     const uint32_t t_row = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const int seg = is_k ? p.dn : p.head_dim;
+    const CUtensorMap* tm_out = is_k ? &tm_ko : &tm_vo;
     __nv_bfloat16* out = is_k ? p.k : p.v;
-    const int chunks = n_valid / 8;  // 16-byte pieces per staged row
-    // output offset of chunk ch of this column tile: head h = col / seg and
-    // column e = col % seg (seg % 8 == 0: no chunk straddles two heads)
-    if (et < chunks) {
-      const int col = col0 + et * 8;
-      col_off[et] = static_cast<long long>(col / seg) * p.slots * p.head_dim + col % seg;
-    }
+    const int boxes = n_valid / 32;  // staged 32-column boxes (n_valid is a multiple of 32)
     // heads whose key rows start in this tile: offsets of their positional part
     int n_heads = 0;
     if (is_k && p.d_r > 0)
-      for (int ch = 0; ch < chunks; ++ch)
+      for (int ch = 0; ch < n_valid / 8; ++ch)
         if ((col0 + ch * 8) % seg == 0) {
           if (et == 0)
             head_off[n_heads] =
@@ -217,12 +221,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++n_heads;
         }
     const int kr_chunks = p.d_r / 8;  // 16-byte pieces of one positional key (<= 8)
-    // this thread's first (row, chunk) in the cooperative store loop and the step
-    const int row0 = et / chunks, ch0 = et % chunks;
-    const int drow = kEpiThreads / chunks, dch = kEpiThreads % chunks;
     for (int i = 0, r = g; r < p.n_row_tiles; ++i, r += G) {
       const int s = i & 1;
-      // positional keys of this tile's slots: piece u = et + 256 k is piece
+      const int bb = r / p.tiles_per_b;
+      const int sl0 = (r % p.tiles_per_b) * kBM;  // first slot of the tile
+      // positional keys of this tile's slots: piece u = et + 384 k is piece
       // u % kr_chunks of row u / kr_chunks (coalesced), loaded ahead of use
       constexpr int kKr = (kBM * 8 + kEpiThreads - 1) / kEpiThreads;
       uint4 krv[kKr];
@@ -230,56 +233,50 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int k = 0; k < kKr; ++k) {
           const int u = et + kEpiThreads * k, row = u / kr_chunks;
-          const int m = r * kBM + row;
-          if (u < kBM * kr_chunks && m < p.M)
-            krv[k] = __ldg(reinterpret_cast<const uint4*>(p.kr + static_cast<size_t>(m) * p.d_r) +
+          if (u < kBM * kr_chunks && sl0 + row < p.slots)
+            krv[k] = __ldg(reinterpret_cast<const uint4*>(
+                               p.kr + (static_cast<size_t>(bb) * p.slots + sl0 + row) * p.d_r) +
                            u % kr_chunks);
         }
       }
       const bool got = mbar_wait(&acc_full[s], (i >> 1) & 1, wc) && !*abort_flag;
       if (got) {
         tc_fence_after();
-        uint8_t* srow = stage_out + rl * S::kOutStride;
+        // row rl of box cb, 64-byte swizzle: 16-byte chunk j at j ^ ((rl >> 1) & 3)
+        const uint32_t sw = static_cast<uint32_t>((rl >> 1) & 3);
 #pragma unroll 1
         for (int cb = part; cb < BN / 32; cb += kParts) {
           uint32_t v[32];
           tmem_ld32(t_row + s * BN + cb * 32, v);
           tmem_wait_ld();
-          uint32_t pk[16];
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            pk[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+          uint8_t* brow = stage_out + cb * S::kBoxBytes + rl * 64;
 #pragma unroll
           for (int j = 0; j < 4; ++j)
-            *reinterpret_cast<uint4*>(srow + cb * 64 + j * 16) =
-                make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+            *reinterpret_cast<uint4*>(brow + ((j ^ sw) << 4)) =
+                make_uint4(pack_bf16x2(__uint_as_float(v[8 * j]), __uint_as_float(v[8 * j + 1])),
+                           pack_bf16x2(__uint_as_float(v[8 * j + 2]), __uint_as_float(v[8 * j + 3])),
+                           pack_bf16x2(__uint_as_float(v[8 * j + 4]), __uint_as_float(v[8 * j + 5])),
+                           pack_bf16x2(__uint_as_float(v[8 * j + 6]), __uint_as_float(v[8 * j + 7])));
         }
       }
-      if (part == 0) {  // offset of slot row rl's output row (batch, head 0, slot), -1 past the end
-        const int m = r * kBM + rl;
-        const int bb = m / p.slots, sl = m - bb * p.slots;
-        row_base[rl] = m < p.M ? (static_cast<long long>(bb) * p.heads * p.slots + sl) * p.head_dim
-                               : -1ll;
-      }
+      if (part == 0)  // output offset of slot row rl (batch, head 0, slot), -1 past the last slot
+        row_base[rl] = sl0 + rl < p.slots
+                           ? (static_cast<long long>(bb) * p.heads * p.slots + sl0 + rl) * p.head_dim
+                           : -1ll;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[s]);
+      fence_proxy_async_smem();       // the staged boxes reach the TMA stores
       if (!epilogue_all(got)) break;  // staged tile complete, or every thread leaves
-      int row = row0, ch = ch0;
-#pragma unroll 4
-      for (int q = et; q < kBM * chunks; q += kEpiThreads) {
-        const long long rb = row_base[row];
-        if (rb >= 0 && debug_in_range(rb + col_off[ch], 0,
-                                      static_cast<long long>(p.M) * p.heads * p.head_dim - 7,
-                                      p.status))
-          *reinterpret_cast<uint4*>(out + rb + col_off[ch]) =
-              *reinterpret_cast<const uint4*>(stage_out + row * S::kOutStride + ch * 16);
-        row += drow;
-        ch += dch;
-        if (ch >= chunks) {
-          ch -= chunks;
-          ++row;
+      if (et == 0) {
+        // one tensor store per box: columns col .. col + 31 are columns e .. e + 31
+        // of head h, slots sl0 .. sl0 + 127 of batch element bb
+        for (int bx = 0; bx < boxes; ++bx) {
+          const int col = col0 + bx * 32;
+          tma_store_3d(tm_out, stage_out + bx * S::kBoxBytes, col % seg, sl0,
+                       bb * p.heads + col / seg);
         }
+        bulk_commit();
       }
       if (n_heads > 0) {
 #pragma unroll
@@ -293,7 +290,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     krv[k];
         }
       }
-      epilogue_sync();  // staging free for the next tile
+      if (et == 0) bulk_wait_read_all();  // the stores have read the staged boxes
+      epilogue_sync();                    // staging free for the next tile
     }
   }
 
@@ -311,12 +309,18 @@ int launch_dec(const DecompressArgs& a) {
   const int dn = a.head_dim - a.d_r;
   const unsigned long long M = static_cast<unsigned long long>(a.batch) * a.slots;
   const int cols_k = a.heads * dn, cols_v = a.heads * a.head_dim;
-  CUtensorMap tm_c, tm_wk, tm_wv;
+  CUtensorMap tm_c, tm_wk, tm_wv, tm_ko, tm_vo;
+  // outputs as [batch * heads][slots][head_dim], written in [128 x 32] boxes
+  const unsigned long long HD = a.head_dim, SL = a.slots;
   if (!encode_map_2d_bf16(&tm_c, a.c, DC, M, DC * 2ull, 64, kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_wk, a.w_uk, DC, cols_k, DC * 2ull, 64, S::BN,
                           CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_wv, a.w_uv, DC, cols_v, DC * 2ull, 64, S::BN,
-                          CU_TENSOR_MAP_SWIZZLE_128B))
+                          CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_map_3d_bf16(&tm_ko, a.k, HD, SL, static_cast<unsigned long long>(a.batch) * a.heads,
+                          HD * 2, SL * HD * 2, 32, kBM, CU_TENSOR_MAP_SWIZZLE_64B) ||
+      !encode_map_3d_bf16(&tm_vo, a.v, HD, SL, static_cast<unsigned long long>(a.batch) * a.heads,
+                          HD * 2, SL * HD * 2, 32, kBM, CU_TENSOR_MAP_SWIZZLE_64B))
     return MLA_ERR_CUDA;
   auto kern = mla_decompress_tc_kernel<DC>;
   cudaError_t e =
@@ -330,7 +334,8 @@ int launch_dec(const DecompressArgs& a) {
   kp.k = static_cast<__nv_bfloat16*>(a.k);
   kp.v = static_cast<__nv_bfloat16*>(a.v);
   kp.M = static_cast<int>(M);
-  kp.n_row_tiles = static_cast<int>((M + kBM - 1) / kBM);
+  kp.tiles_per_b = (a.slots + kBM - 1) / kBM;  // a tile never spans two batch elements
+  kp.n_row_tiles = kp.tiles_per_b * a.batch;
   kp.tiles_k = (cols_k + S::BN - 1) / S::BN;
   kp.cols_k = cols_k;
   kp.cols_v = cols_v;
@@ -348,7 +353,8 @@ int launch_dec(const DecompressArgs& a) {
   int groups = sms / n_col;
   if (groups < 1) groups = 1;
   if (groups > kp.n_row_tiles) groups = kp.n_row_tiles;
-  kern<<<dim3(n_col, groups), kThreads, S::kSmemBytes, a.stream>>>(tm_c, tm_wk, tm_wv, kp);
+  kern<<<dim3(n_col, groups), kThreads, S::kSmemBytes, a.stream>>>(tm_c, tm_wk, tm_wv, tm_ko,
+                                                                     tm_vo, kp);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
@@ -361,7 +367,8 @@ int launch_dec(const DecompressArgs& a) {
 
 int launch_decompress(const DecompressArgs& a) {
   const int dn = a.head_dim - a.d_r;
-  if (dn <= 0 || dn % 8 != 0 || a.head_dim % 8 != 0 || a.d_r % 8 != 0)
+  // whole 32-column output boxes, none spanning two heads
+  if (dn <= 0 || dn % 32 != 0 || a.head_dim % 32 != 0 || a.d_r % 8 != 0)
     return MLA_ERR_UNSUPPORTED;
   if (static_cast<long long>(a.batch) * a.slots >= (1ll << 31)) return MLA_ERR_UNSUPPORTED;
   switch (a.d_c) {
