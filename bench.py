@@ -760,6 +760,43 @@ def run_sweep(args):
             "sweep": rows}
 
 
+# ------------------------------------------------- the other configs, briefly
+def other_configs():
+    """The benchmark's other configurations, each measured in its own short
+    timed region of the default run, so that one bench line covers them all:
+    the tiny single layer (config 1), the 30-layer step (config 3), the batch-4
+    rollout window (config 4) and the d_c x d_r sweep next to the dense
+    baseline (config 5). Fewer steps than their own commands
+    (`--workload tiny|wan30|rollout`, `--sweep dc`); a configuration that fails
+    records its error instead of stopping the line."""
+    res = {}
+    for key, name, steps in (("config1_tiny", "tiny", 50), ("config3_wan30", "wan30", 5),
+                             ("config4_rollout", "rollout", 20)):
+        try:
+            ns = argparse.Namespace(steps=steps, warmup=3, no_cpu_baseline=True, cpu_budget=0.0)
+            o = run_ours(ns, synth.workload(name))
+            res[key] = {"workload": o["config"]["workload"], "steps": steps,
+                        "ms_per_step": o["ms_per_step"], "value": o["value"], "unit": o["unit"],
+                        "attention_frac_of_peak": o["roofline"]["frac"],
+                        "peak_source": o["roofline"]["peak_source"],
+                        "append_frac_of_hbm": o["roofline_append"]["frac"],
+                        "e2e": o["e2e"]["value"], "sm_mhz": o["clocks"].get("sm_mhz")}
+        except Exception as e:  # noqa: BLE001 - recorded in the line
+            res[key] = {"error": f"{type(e).__name__}: {e}"[:300]}
+        torch.cuda.empty_cache()
+    try:
+        sw = run_sweep(argparse.Namespace(steps=10, warmup=3))
+        res["config5_sweep"] = {
+            "steps": 10, "unit": "ms per chunk per layer",
+            "rows": [{k: r[k] for k in ("layout", "d_c", "d_r", "ms_per_chunk_layer", "tflops",
+                                        "frac_of_measured_bf16_burst") if k in r}
+                     for r in sw["sweep"]]}
+    except Exception as e:  # noqa: BLE001
+        res["config5_sweep"] = {"error": f"{type(e).__name__}: {e}"[:300]}
+    torch.cuda.empty_cache()
+    return res
+
+
 # ------------------------------------------------------------- crossover
 def run_crossover(args):
     """Absorbed attention (App. E) against decompress-then-dense (Eq.
@@ -1053,6 +1090,9 @@ def main():
                          "phase; crossover: absorbed vs decompress-then-dense by chunk size "
                          "(one JSON line each)")
     ap.add_argument("--mem-budget-gb", type=float, default=B200_USABLE_GB)
+    ap.add_argument("--no-other-configs", action="store_true",
+                    help="skip the brief measurements of configs 1, 3, 4 and 5 that the "
+                         "default run adds to its line")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -1083,6 +1123,8 @@ def main():
         out = run_reference(args, w)
     else:
         out = run_ours(args, w)
+        if args.workload == "wan" and not args.no_other_configs:
+            out["other_configs"] = other_configs()
     print(json.dumps(out), flush=True)
 
 
