@@ -51,13 +51,14 @@ struct DecShape {
   static constexpr int kStageOff = kWBytes + 2 * kCBytes;
   static constexpr int kBarOff = kStageOff + (BN / 32) * kBoxBytes;
   // per-row output offsets of the positional-key copies
-  static constexpr int kRowTabOff = kBarOff + 128;             // long long [128]
-  static constexpr int kHeadTabOff = kRowTabOff + kBM * 8;     // long long [BN/8]
+  static constexpr int kRowTabOff = kBarOff + 128;             // long long [2][128]
+  static constexpr int kHeadTabOff = kRowTabOff + 2 * kBM * 8;  // long long [BN/8]
   static constexpr int kSmemBytes = 1024 + kHeadTabOff + (BN / 8) * 8;
   static constexpr uint32_t kTmemCols = 2 * BN <= 256 ? 256 : 512;
   static constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, BN, false, false);
   static_assert(DC % 64 == 0 && DC <= 256, "latent width");
-  static_assert(BN % 32 == 0 && BN <= 256, "tile width: whole 32-column boxes");
+  static_assert(BN % 32 == 0 && BN <= 256 && (BN / 32) % kParts == 0 && BN / 32 <= 2 * kParts,
+                "tile width: whole 32-column boxes, one or two per epilogue warp");
   static_assert(kChunkBytesW % 1024 == 0 && kStageOff % 1024 == 0, "swizzle-atom alignment");
   static_assert(kSmemBytes <= 232448, "shared memory");
 };
@@ -210,6 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const CUtensorMap* tm_out = is_k ? &tm_ko : &tm_vo;
     __nv_bfloat16* out = is_k ? p.k : p.v;
     const int boxes = n_valid / 32;  // staged 32-column boxes (n_valid is a multiple of 32)
+    constexpr int kPhases = BN / 32 / kParts;  // boxes per epilogue warp: 2 (BN = 192) or 1
     // heads whose key rows start in this tile: offsets of their positional part
     int n_heads = 0;
     if (is_k && p.d_r > 0)
@@ -240,59 +242,81 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       const bool got = mbar_wait(&acc_full[s], (i >> 1) & 1, wc) && !*abort_flag;
-      if (got) {
-        tc_fence_after();
-        // row rl of box cb, 64-byte swizzle: 16-byte chunk j at j ^ ((rl >> 1) & 3)
-        const uint32_t sw = static_cast<uint32_t>((rl >> 1) & 3);
-#pragma unroll 1
-        for (int cb = part; cb < BN / 32; cb += kParts) {
-          uint32_t v[32];
-          tmem_ld32(t_row + s * BN + cb * 32, v);
-          tmem_wait_ld();
-          uint8_t* brow = stage_out + cb * S::kBoxBytes + rl * 64;
+      if (got) tc_fence_after();
+      // row rl of box cb, 64-byte swizzle: 16-byte chunk j at j ^ ((rl >> 1) & 3)
+      const uint32_t sw = static_cast<uint32_t>((rl >> 1) & 3);
+      auto stage_box = [&](int cb) {
+        uint32_t v[32];
+        tmem_ld32(t_row + s * BN + cb * 32, v);
+        tmem_wait_ld();
+        uint8_t* brow = stage_out + cb * S::kBoxBytes + rl * 64;
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            *reinterpret_cast<uint4*>(brow + ((j ^ sw) << 4)) =
-                make_uint4(pack_bf16x2(__uint_as_float(v[8 * j]), __uint_as_float(v[8 * j + 1])),
-                           pack_bf16x2(__uint_as_float(v[8 * j + 2]), __uint_as_float(v[8 * j + 3])),
-                           pack_bf16x2(__uint_as_float(v[8 * j + 4]), __uint_as_float(v[8 * j + 5])),
-                           pack_bf16x2(__uint_as_float(v[8 * j + 6]), __uint_as_float(v[8 * j + 7])));
-        }
-      }
-      if (part == 0)  // output offset of slot row rl (batch, head 0, slot), -1 past the last slot
-        row_base[rl] = sl0 + rl < p.slots
-                           ? (static_cast<long long>(bb) * p.heads * p.slots + sl0 + rl) * p.head_dim
-                           : -1ll;
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[s]);
-      fence_proxy_async_smem();       // the staged boxes reach the TMA stores
-      if (!epilogue_all(got)) break;  // staged tile complete, or every thread leaves
-      if (et == 0) {
-        // one tensor store per box: columns col .. col + 31 are columns e .. e + 31
-        // of head h, slots sl0 .. sl0 + 127 of batch element bb
-        for (int bx = 0; bx < boxes; ++bx) {
+        for (int j = 0; j < 4; ++j)
+          *reinterpret_cast<uint4*>(brow + ((j ^ sw) << 4)) =
+              make_uint4(pack_bf16x2(__uint_as_float(v[8 * j]), __uint_as_float(v[8 * j + 1])),
+                         pack_bf16x2(__uint_as_float(v[8 * j + 2]), __uint_as_float(v[8 * j + 3])),
+                         pack_bf16x2(__uint_as_float(v[8 * j + 4]), __uint_as_float(v[8 * j + 5])),
+                         pack_bf16x2(__uint_as_float(v[8 * j + 6]), __uint_as_float(v[8 * j + 7])));
+      };
+      // one tensor store per box: columns col .. col + 31 are columns e .. e + 31
+      // of head h, slots sl0 .. sl0 + 127 of batch element bb
+      auto store_boxes = [&](int bx0, int bx1) {
+        for (int bx = bx0; bx < bx1 && bx < boxes; ++bx) {
           const int col = col0 + bx * 32;
           tma_store_3d(tm_out, stage_out + bx * S::kBoxBytes, col % seg, sl0,
                        bb * p.heads + col / seg);
         }
         bulk_commit();
+      };
+      long long* rbase = row_base + (i & 1) * kBM;  // read by this tile's key copies
+      if (part == 0)  // output offset of slot row rl (batch, head 0, slot), -1 past the last slot
+        rbase[rl] = sl0 + rl < p.slots
+                        ? (static_cast<long long>(bb) * p.heads * p.slots + sl0 + rl) * p.head_dim
+                        : -1ll;
+      if constexpr (kPhases == 1) {
+        if (got) stage_box(part);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[s]);
+        fence_proxy_async_smem();       // the staged boxes reach the TMA stores
+        if (!epilogue_all(got)) break;  // staged tile complete, or every thread leaves
+        if (et == 0) store_boxes(0, BN / 32);
+      } else {
+        // two phases over the boxes (each part's first box, then its second),
+        // so that one phase's stores read shared memory while the other phase
+        // is staged
+        if (got) stage_box(part);
+        fence_proxy_async_smem();
+        if (et == 0) bulk_wait_read_all();  // the last tile's second-phase boxes are free
+        if (!epilogue_all(got)) break;      // first-phase boxes staged
+        if (et == 0) store_boxes(0, kParts);
+        if (got) stage_box(part + kParts);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[s]);
+        fence_proxy_async_smem();
+        if (et == 0) bulk_wait_read_all();  // this tile's first-phase boxes are free again
+        epilogue_sync();                    // second-phase boxes staged
+        if (et == 0) store_boxes(kParts, 2 * kParts);
       }
       if (n_heads > 0) {
 #pragma unroll
         for (int k = 0; k < kKr; ++k) {
           const int u = et + kEpiThreads * k, row = u / kr_chunks;
-          if (u < kBM * kr_chunks && row_base[row] >= 0)
+          if (u < kBM * kr_chunks && rbase[row] >= 0)
             for (int a = 0; a < n_heads; ++a)
-              if (debug_in_range(row_base[row] + head_off[a] + 8 * (u % kr_chunks), 0,
+              if (debug_in_range(rbase[row] + head_off[a] + 8 * (u % kr_chunks), 0,
                                  static_cast<long long>(p.M) * p.heads * p.head_dim - 7, p.status))
-                *reinterpret_cast<uint4*>(out + row_base[row] + head_off[a] + 8 * (u % kr_chunks)) =
+                *reinterpret_cast<uint4*>(out + rbase[row] + head_off[a] + 8 * (u % kr_chunks)) =
                     krv[k];
         }
       }
-      if (et == 0) bulk_wait_read_all();  // the stores have read the staged boxes
-      epilogue_sync();                    // staging free for the next tile
+      if constexpr (kPhases == 1) {
+        if (et == 0) bulk_wait_read_all();  // the stores have read the staged boxes
+        epilogue_sync();                    // staging free for the next tile
+      }
     }
+    if (et == 0) bulk_wait_read_all();
   }
 
   tc_fence_before();
