@@ -27,8 +27,7 @@
 //              softmax: thread i owns row i, copies S_j out of TMEM (releasing
 //              it), writes P_j (bf16) once PV_{j-1} has read the previous P,
 //              rescales O in TMEM only when its running max grows by more
-//              than 2^8, and finally stages O / l as bf16 rows in the freed
-//              key stages, from which one bulk copy writes the row tile.
+//              than 2^8, and finally writes O / l as bf16.
 // TMEM columns: S [0,BN) P [BN,3BN/2) O [3BN/2,3BN/2+d_c) Q [3BN/2+d_c, +(d_c+d_r)/2).
 // When Q does not fit there (d_c = 256) it stays in shared memory (TMA-loaded
 // q_c plus the rotated q_r stored by the softmax warps) and QK reads it there;
