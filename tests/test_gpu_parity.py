@@ -111,10 +111,15 @@ def test_append_parity_ragged_batch2_wrap():
     assert_close(f64(cache.kr)[:, valid], oc.kr[:, valid], what="k_rope")
 
 
-def test_ring_bit_exact():
+@pytest.mark.parametrize("batch", [2, 64, 160])
+def test_ring_bit_exact(batch):
     """One-hot projections, no RMSNorm, positions at zero: every appended
-    value is an input value, so slot contents must match bit for bit."""
-    w = small(grid_h=6, grid_w=7, window_frames=4, batch=2)
+    value is an input value, so slot contents must match bit for bit. With
+    42 tokens per frame a token tile holds several frames (slot runs break
+    inside tiles, the ring wraps inside tiles). Batch 2 takes the append's
+    cluster form, 64 one CTA per tile, 160 (more tiles than SMs) two CTAs
+    per SM."""
+    w = small(grid_h=6, grid_w=7, window_frames=4, batch=batch)
     cfg = V.make_config(w, V.MLA_FLAG_NO_RMSNORM)
     cache = V.LatentCache(cfg)
     V.mla_cache_reset(cache)

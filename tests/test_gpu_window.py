@@ -78,13 +78,16 @@ SINK_SCHEDULES = [
 
 
 @pytest.mark.parametrize("sched", range(len(SINK_SCHEDULES)))
-@pytest.mark.parametrize("flags", [0, V.MLA_FLAG_SIMT])
-def test_sink_fifo_slots_bit_exact(flags, sched):
+@pytest.mark.parametrize("flags,batch", [(0, 2), (V.MLA_FLAG_SIMT, 2), (0, 64), (0, 160)])
+def test_sink_fifo_slots_bit_exact(flags, batch, sched):
     """One-hot projections, no RMSNorm: every stored value is an input value,
     so the sink + FIFO slot map and the unrotated k^R match bit for bit. An
-    append of more than W - S frames past the sinks is refused."""
+    append of more than W - S frames past the sinks is refused. Batches 2, 64
+    and 160 take the tensor-core append's cluster, one-CTA-per-tile and
+    two-CTAs-per-SM forms (slot runs break at the sink boundary and the FIFO
+    wrap inside token tiles)."""
     schedule, expect_held = SINK_SCHEDULES[sched]
-    w = synth.workload("tiny", grid_h=6, grid_w=7, window_frames=4, sink_frames=1, batch=2)
+    w = synth.workload("tiny", grid_h=6, grid_w=7, window_frames=4, sink_frames=1, batch=batch)
     cfg = V.make_config(w, flags | V.MLA_FLAG_NO_RMSNORM)
     assert cfg.flags & V.MLA_FLAG_ROTATE_AT_USE
     cache = V.LatentCache(cfg)
