@@ -64,8 +64,9 @@ __device__ __forceinline__ void debug_count_rescale(bool rescaled, int* status) 
 // Programmatic dependent launch. The library's kernels are launched with
 // programmatic stream serialization, so their CTAs may start while the
 // previous kernel in the stream is still running. Before grid_dep_sync() a
-// kernel only does set-up that touches no global memory (barrier init, TMEM
-// allocation, cluster sync); grid_dep_sync() lets the next kernel in the
+// kernel only does set-up (barrier init, TMEM allocation, cluster sync) and
+// L2 prefetches, which read nothing into the SM and store nothing;
+// grid_dep_sync() lets the next kernel in the
 // stream launch once every CTA of this one has started, then waits until the
 // previous kernel has completed and its writes are visible. Every thread
 // calls it before its first global-memory access.
@@ -184,6 +185,21 @@ __device__ __forceinline__ void tma_load_3d(void* smem_dst, const CUtensorMap* m
       " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(smem_dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
       : "memory");
+}
+// Warm L2 with a box of a rank-3 or rank-2 tensor (no shared memory, no
+// barrier, no result). L2 is the one place where the GPU's accesses to device memory
+// meet, so a line warmed before another kernel writes it is updated there,
+// and a later copy reads the written data.
+__device__ __forceinline__ void tma_prefetch_l2_3d(const CUtensorMap* map, int c0, int c1,
+                                                   int c2) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int c0, int c1) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1)
+               : "memory");
 }
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar,
                                             int c0, int c1) {
