@@ -38,14 +38,13 @@ constexpr int kThreads = 192;
 // CTAs sharing an SM (228 KB per SM, 1 KB of it reserved per CTA)
 constexpr int kSmemOne = 232448;
 constexpr int kSmemHalf = (233472 - 2 * 1024) / 2;
-// K blocks of x each CTA warms into L2 before the wait for the previous
-// kernel: CTAs of the first wave (which start while that kernel finishes,
-// HBM being mostly idle) and later ones (which start under this kernel's own
-// K loops); the two-CTAs-per-SM form holds two stages per CTA and profits
-// from a deeper first prefetch
+// K blocks of x a CTA of the first wave warms into L2 before its wait for
+// the previous kernel (those CTAs start while that kernel finishes, HBM being
+// mostly idle; later ones start under this kernel's own K loops and warm
+// nothing). The two-CTAs-per-SM form holds two stages per CTA and profits
+// from a deeper prefetch.
 constexpr int kPrefetchOne = 4;
-constexpr int kPrefetchX2First = 12;
-constexpr int kPrefetchX2Later = 4;
+constexpr int kPrefetchX2 = 12;
 
 // What one CTA computes: NC columns of c, from column c0 (given at run time),
 // and NK columns of k^R, into one [128 x (NC + NK)] TMEM accumulator:
@@ -110,8 +109,8 @@ struct AppendKParams {
   int rope_len, pairs_t, pairs_h, use_rmsnorm, rotate;
   float eps;
   int* status;
-  int first_wave;           // CTAs resident at once (linear block index below it: first wave)
-  int pf_first, pf_later;   // x K blocks warmed into L2 by a first-wave / later CTA
+  int first_wave;  // CTAs resident at once (a linear block index below it: the first wave)
+  int pf_blocks;   // x K blocks a first-wave CTA warms into L2
 };
 
 // tile: the token tile (128 tokens) of this CTA; c0: its first column of c
@@ -159,20 +158,21 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   constexpr uint16_t kAll = static_cast<uint16_t>((1u << CL) - 1u);
   const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   // While the previous kernel in the stream finishes, HBM is mostly idle:
-  // the first x boxes of this CTA's tile (its part of them in a cluster) are
-  // warmed into L2 then, so that the K loop starts on L2 hits. Only the
-  // copies into shared memory wait for the previous kernel.
-  // The weights are shared by every tile: each CTA warms this slice's rows
-  // of one K block, so that the first CTAs' copies do not all miss together.
-  if (warp == 0 && lane == 0 && crank < S::kXParts) {
-    const long long lin =
-        blockIdx.x + static_cast<long long>(gridDim.x) * (blockIdx.y + gridDim.y * blockIdx.z);
-    const int depth = lin < p.first_wave ? p.pf_first : p.pf_later;
-    const int kpf = p.k_blocks < depth ? p.k_blocks : depth;
+  // a CTA of the first wave warms the first x boxes of its tile (its part of
+  // them in a cluster) into L2 then, so that the K loop starts on L2 hits.
+  // Only the copies into shared memory wait for the previous kernel. The
+  // weights are shared by every tile: each first-wave CTA also warms its
+  // slice's rows of one K block, so that the first copies do not all miss
+  // together.
+  const long long lin =
+      blockIdx.x + static_cast<long long>(gridDim.x) * (blockIdx.y + gridDim.y * blockIdx.z);
+  const bool first_wave = lin < p.first_wave;
+  if (first_wave && warp == 0 && lane == 0 && crank < S::kXParts) {
+    const int kpf = p.k_blocks < p.pf_blocks ? p.k_blocks : p.pf_blocks;
     for (int kb = 0; kb < kpf; ++kb)
       tma_prefetch_l2_3d(tm_x, kb * kBK, row0 + crank * S::kXRows, b);
   }
-  if (warp == 0 && lane == 1) {
+  if (first_wave && warp == 0 && lane == 1) {
     const int kb = (tile + static_cast<int>(gridDim.x) * b) % p.k_blocks;
     if constexpr (NC > 0)
       for (int h = 0; h < NC / S::kWcBox; ++h)
@@ -613,8 +613,7 @@ int launch_tc(const AppendArgs& a) {
   kp.eps = a.eps;
   kp.status = a.status;
   kp.first_wave = sms * (x2 ? 2 : 1);
-  kp.pf_first = x2 ? kPrefetchX2First : kPrefetchOne;
-  kp.pf_later = x2 ? kPrefetchX2Later : kPrefetchOne;
+  kp.pf_blocks = x2 ? kPrefetchX2 : kPrefetchOne;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(cluster ? tiles * kCl : tiles, a.batch, kSplit ? 2 : 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
