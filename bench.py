@@ -14,7 +14,7 @@ one JSON line each: the latent-size sweep next to the dense baseline, the
 memory-cap batch sweep, the whole layer by phase, and absorbed vs
 decompress-then-dense by query-chunk size.
 
-Single GPU only. Every tensor-core kernel shares tiles among the CTAs of a
+Single GPU only. The attention kernels share key tiles among the CTAs of a
 cluster by TMA multicast within this GPU's memory, which may only run in
 single-GPU jobs; under torchrun with more than one rank the GPU arm prints an
 "unavailable" line (rank 0) and every rank exits 0. The reference arm (the
@@ -1066,7 +1066,7 @@ def run_memcap(args):
 
 # ----------------------------------------------------------------- helpers
 PIPE_FLOP_PER_CLK_SM = 8192  # measured tcgen05 bf16 rate per SM (N = 128..256)
-MULTI_GPU_CLOSED = ("multi-GPU runs are closed on this pool: every tensor-core kernel shares "
+MULTI_GPU_CLOSED = ("multi-GPU runs are closed on this pool: the attention kernels share key "
                     "tiles among the CTAs of a cluster by TMA multicast, which may only run in "
                     "single-GPU jobs")
 

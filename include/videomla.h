@@ -10,8 +10,9 @@
  *  - Every buffer must be device memory (cudaMalloc or a pool built on it)
  *    of the CURRENT device: host memory, pinned or not, managed memory and
  *    another GPU's memory are refused with MLA_ERR_ARG before any launch.
- *    The kernels copy tiles with TMA and share them among the CTAs of a
- *    cluster by multicast, which addresses this GPU's own memory only.
+ *    The kernels copy tiles with TMA, and the attention kernels share key
+ *    tiles among the CTAs of a cluster by multicast, which addresses this
+ *    GPU's own memory only.
  *  - The library caches, per device, the device addresses of its two
  *    file-scope arrays (the status word and the no-allocation scratch). It
  *    does not survive cudaDeviceReset (or any other teardown of the

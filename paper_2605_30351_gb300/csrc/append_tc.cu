@@ -55,9 +55,10 @@ constexpr int kPrefetchX2 = 12;
 //  - a grid too small to occupy the SMs (one chunk at batch 1): a cluster
 //    of CL = d_c/64 CTAs per token tile, one per 64 columns of c, the last
 //    also computing k^R, so that each SM streams the token tile and only its
-//    share of the weights. The CTAs share each x box through TMA multicast
-//    (each fetches a part of it from L2 for all) and exchange their partial
-//    RMSNorm sums of squares through distributed shared memory.
+//    share of the weights. Every CTA fetches the whole x box (from L2 after
+//    the first), so the CTAs' K loops do not wait on one another; they
+//    exchange their partial RMSNorm sums of squares through distributed
+//    shared memory.
 template <int DC, int DR, int NC, int NK, int CL = 1, int BUDGET = kSmemOne>
 struct AppendShape {
   static constexpr int N = NC + NK;
@@ -65,13 +66,11 @@ struct AppendShape {
   static constexpr int kWcBox = NC == 0 ? 64 : (NC < 256 ? NC : 256);  // W_dkv rows per TMA box
   static constexpr int kABytes = kBM * kBK * 2;
   // rows of a stage's weight region: in a cluster every CTA takes the widest
-  // slice's layout, so that multicast copies and barriers sit at the same
-  // offsets in all of them
+  // slice's layout (one shared-memory size for the launch, and the partial
+  // sums at the same offset in every CTA)
   static constexpr int kBRows = CL > 1 ? 64 + DR : N;
   static constexpr int kBBytes = kBRows * kBK * 2;
   static constexpr int kTxBytes = kABytes + N * kBK * 2;  // lands in this CTA per stage
-  static constexpr int kXParts = CL == 3 ? 2 : CL;       // ranks fetching a part of each x box
-  static constexpr int kXRows = kBM / kXParts;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kBarBytes = 256;
   // [CL][128] partial sums of squares at the front of shared memory: the same
@@ -93,8 +92,7 @@ struct AppendShape {
                     (CL == DC / 64 && CL >= 2 && DC <= 256 && NC == 64),
                 "parts are split for d_c > 256, or over a cluster of 64-column slices");
   static_assert(N <= 512, "accumulator must fit in TMEM");
-  static_assert(kStageBytes % 1024 == 0 && (kXRows * 128) % 1024 == 0, "swizzle-atom alignment");
-  static_assert(kXParts * kXRows == kBM && kWcBox > 0, "x box split over the cluster");
+  static_assert(kStageBytes % 1024 == 0 && kWcBox > 0, "swizzle-atom alignment");
   static_assert(kStages >= 2, "smem");
 };
 
@@ -141,7 +139,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   if (threadIdx.x == 0) {
     for (int s = 0; s < NST; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], CL);  // released by the MMA of every CTA of the cluster
+      mbar_init(&empty[s], 1);
     }
     mbar_init(acc_full, 1);
     *abort_flag = 0;
@@ -155,7 +153,6 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  constexpr uint16_t kAll = static_cast<uint16_t>((1u << CL) - 1u);
   const int crank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   // While the previous kernel in the stream finishes, HBM is mostly idle:
   // a CTA of the first wave warms the first x boxes of its tile (its part of
@@ -167,10 +164,9 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
   const long long lin =
       blockIdx.x + static_cast<long long>(gridDim.x) * (blockIdx.y + gridDim.y * blockIdx.z);
   const bool first_wave = lin < p.first_wave;
-  if (first_wave && warp == 0 && lane == 0 && crank < S::kXParts) {
+  if (first_wave && warp == 0 && lane == 0 && crank == 0) {
     const int kpf = p.k_blocks < p.pf_blocks ? p.k_blocks : p.pf_blocks;
-    for (int kb = 0; kb < kpf; ++kb)
-      tma_prefetch_l2_3d(tm_x, kb * kBK, row0 + crank * S::kXRows, b);
+    for (int kb = 0; kb < kpf; ++kb) tma_prefetch_l2_3d(tm_x, kb * kBK, row0, b);
   }
   if (first_wave && warp == 0 && lane == 1) {
     const int kb = (tile + static_cast<int>(gridDim.x) * b) % p.k_blocks;
@@ -179,7 +175,8 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
         tma_prefetch_l2_2d(tm_wc, kb * kBK, c0 + h * S::kWcBox);
     if constexpr (NK > 0) tma_prefetch_l2_2d(tm_wk, kb * kBK, 0);
   }
-  // every CTA's barriers must be initialised before a peer's multicast lands
+  // every CTA of the cluster has started before a peer writes its shared
+  // memory (the partial sums of squares)
   if constexpr (CL > 1) cluster_sync();
   grid_dep_sync();
 
@@ -195,26 +192,13 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
         uint8_t* a = smem + st * S::kStageBytes;
         uint8_t* bm = a + S::kABytes;
         mbar_arrive_expect_tx(&full[st], S::kTxBytes);
-        if constexpr (CL > 1) {
-          // this rank's rows of the x box, multicast to every CTA of the cluster
-          if (crank < S::kXParts)
-            tma_load_3d_mc(a + crank * S::kXRows * 128, tm_x, &full[st], kb * kBK,
-                           row0 + crank * S::kXRows, b, kAll);
-        } else {
-          tma_load_3d(a, tm_x, &full[st], kb * kBK, row0, b);
-        }
+        tma_load_3d(a, tm_x, &full[st], kb * kBK, row0, b);
         if constexpr (NC > 0)
           for (int h = 0; h < NC / S::kWcBox; ++h)
             tma_load_2d(bm + h * S::kWcBox * 128, tm_wc, &full[st], kb * kBK,
                         c0 + h * S::kWcBox);
         if constexpr (NK > 0) tma_load_2d(bm + NC * 128, tm_wk, &full[st], kb * kBK, 0);
         issued = kb + 1;
-      }
-      if constexpr (CL > 1) {
-        // the peers' MMAs release every stage through this CTA's barriers:
-        // their last releases must have landed before the CTA may exit
-        for (int st = 0; st < NST && st < p.k_blocks && !*abort_flag; ++st)
-          mbar_wait(&empty[st], (((p.k_blocks - st + NST - 1) / NST) - 1) & 1, wc);
       }
       if (*abort_flag)
         for (int u = issued > NST ? issued - NST : 0; u < issued; ++u)
@@ -258,10 +242,7 @@ __device__ __forceinline__ void append_body(const CUtensorMap* tm_x, const CUten
             }
           }
         }
-        if constexpr (CL > 1)
-          umma_commit_mc(&empty[st], kAll);  // the stage's x part came from every rank
-        else
-          umma_commit(&empty[st]);
+        umma_commit(&empty[st]);
       }
       umma_commit(acc_full);
       if (!ok) mbar_wait_drain(acc_full, 0, p.status);
@@ -572,7 +553,7 @@ int launch_tc(const AppendArgs& a) {
   CUtensorMap tm_x, tm_wc, tm_wk;
   const unsigned long long H = a.hidden, n_tok = a.n_tok;
   if (!encode_map_3d_bf16(&tm_x, a.x, H, n_tok, a.batch, H * 2, n_tok * H * 2, kBK,
-                          cluster ? SCc::kXRows : kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+                          kBM, CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_wc, a.w_dkv, H, DC, H * 2, kBK, cluster ? 64 : S::kWcBox,
                           CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_map_2d_bf16(&tm_wk, a.w_kr, H, DR, H * 2, kBK, DR, CU_TENSOR_MAP_SWIZZLE_128B))

@@ -1,4 +1,4 @@
-"""bench.py has no multi-GPU path: every tensor-core kernel shares tiles among
+"""bench.py has no multi-GPU path: the attention kernels share key tiles among
 the CTAs of a cluster by TMA multicast within one GPU's memory, which may only
 run in single-GPU jobs. Under torchrun with two ranks (the environment a
 2-GPU launch gives each process), rank 0 prints one "unavailable" line and
