@@ -62,6 +62,15 @@ def test_roofline_object(line):
     assert "burst" in r["peak_source"] and abs(r["frac"] - r["frac_of_burst"]) < 1e-9
 
 
+def test_append_roofline_object(line):
+    a = line["roofline_append"]
+    assert a["bound"] == "hbm" and a["unit"] == "GB/s"
+    assert abs(a["frac"] - a["achieved"] / a["peak"]) < 1e-6
+    b = a["back_to_back"]
+    assert 0.0 < b["ms"] <= line["append_ms"] * 1.5
+    assert abs(b["frac"] - b["achieved"] / a["peak"]) < 1e-6 and 0.05 < b["frac"] < 1.5
+
+
 def test_cpu_baseline_object(line):
     c = line["cpu_baseline"]
     for k in ("value", "unit", "cores", "kind", "sample"):
