@@ -449,16 +449,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!mbar_wait(&acc_full[buf], (tl >> 1) & 1, wc)) break;
       tc_fence_after();
-      bulk_wait_read_all();  // the previous tile's copy of this row has read it
       float ss_own = 0.f;
       const uint32_t acc = tmem + t_lane + buf * S::kAccStride;
-#pragma unroll 1
+      // the whole row into registers as bf16 pairs first, so that the
+      // accumulator goes back to the MMA issuer before the staged rows wait
+      // for the previous tile's copies
+      uint32_t pk[BN / 64][32];
+#pragma unroll
       for (int sg = 0; sg < BN / 64; ++sg) {
         uint32_t va[32], vb[32];
         tmem_ld32(acc + sg * 64, va);
         tmem_ld32(acc + sg * 64 + 32, vb);
         tmem_wait_ld();
-        uint32_t pk[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           const uint32_t* v = i < 16 ? va : vb;
@@ -469,14 +471,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (col < n_valid) ss_own = fmaf(a0, a0, ss_own);
             if (col + 1 < n_valid) ss_own = fmaf(a1, a1, ss_own);
           }
-          pk[i] = pack_bf16x2(a0 * scale, a1 * scale);
+          pk[sg][i] = pack_bf16x2(a0 * scale, a1 * scale);
         }
-        stage_row<8>(srow + sg * 128, pk, r & 7);
       }
       // this thread's reads of the accumulator are done: release it to the
       // MMA issuer (in the even CTA)
       tc_fence_before();
       mbar_arrive_cluster(dsmem_addr(smem_u32(&acc_empty[buf]), 0));
+      bulk_wait_read_all();  // the previous tile's copy of this row has read it
+#pragma unroll
+      for (int sg = 0; sg < BN / 64; ++sg) stage_row<8>(srow + sg * 128, pk[sg], r & 7);
       if constexpr (EPI == kStoreSq)
         if (m < p.M) p.sq[static_cast<size_t>(n_tile) * p.M + m] = ss_own;
       if (m < p.M) {
