@@ -719,18 +719,19 @@ int launch_query_prologue(const QueryArgs& a) {
   k2.sq_dim = static_cast<float>(a.d_q);
   k2.eps = a.eps;
   k2.status = a.status;
-  // two-stage ring: two CTAs per SM overlap one tile's epilogue with the next
-  // one's loads (measured 48 vs 51 us at one Wan chunk, 138 vs 164 us at four);
-  // large M: the paired-SM form, as for the first GEMM
-  if (!narrow) {
-    rc = launch_gemm_persistent<256, kRowScale>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
-                                                a.d_q, k2, a.stream);
-    if (rc != MLA_ERR_UNSUPPORTED) return rc;
-    return launch_gemm<256, kRowScale, 3, true>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
-                                                a.d_q, k2, a.stream);
-  }
-  return launch_gemm<256, kRowScale, 2>(a.c_tilde, a.w_qcat, M, a.heads * (a.d_c + a.d_r),
-                                        a.d_q, k2, a.stream);
+  // The persistent paired-SM form at every M: its clusters walk more than one
+  // pair tile each even at one Wan chunk (19 x 11 pair tiles), so each
+  // tile's epilogue runs under the next one's MMAs (one chunk: query prologue
+  // 37.7 -> 32.4 us against the two-CTAs-per-SM form; four chunks: 131 ->
+  // 87 us against the non-persistent paired form). If its clusters cannot be
+  // co-resident, the non-persistent forms: a two-stage ring with two CTAs per
+  // SM at small M, paired-SM MMAs at large M.
+  const int nq = a.heads * (a.d_c + a.d_r);
+  rc = launch_gemm_persistent<256, kRowScale>(a.c_tilde, a.w_qcat, M, nq, a.d_q, k2, a.stream);
+  if (rc != MLA_ERR_UNSUPPORTED) return rc;
+  if (!narrow)
+    return launch_gemm<256, kRowScale, 3, true>(a.c_tilde, a.w_qcat, M, nq, a.d_q, k2, a.stream);
+  return launch_gemm<256, kRowScale, 2>(a.c_tilde, a.w_qcat, M, nq, a.d_q, k2, a.stream);
 }
 
 // ---- fixed scratch for mla_query_prologue_noalloc ----
